@@ -1,0 +1,436 @@
+"""Benchmark of the DARB hot path on the FC6/FC7 workload (AlexNet FC layers).
+
+One step = BMWM re-encode of FC6 (4096x9216) and FC7 (4096x4096), bf16
+weights, then darb_spmm of both at batch 1, 16, 64 and 256.  The reported value
+is effective GB/s: the algorithmic bytes of every call in the step (dense W
+read once by the encoder plus the encoded matrix written; for each product the
+kept values, stored offsets, per-row metadata, X read once and Y written once)
+over the device time of the step.  Inputs rotate over several sets of distinct
+buffers whose total is well above the 129 MB L2, so every call reads cold HBM.
+
+Usage: python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference]
+Under torchrun every rank runs its own copy of the workload (independent
+problems, no data-path collective): weak scaling.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+WORKLOAD = "fc6_fc7"
+BATCHES = (1, 16, 64, 256)
+METRIC = ("darb_spmm effective GB/s & % of HBM roofline at batch 1/16/64/256; encode GB/s")
+NSETS = 4
+FALLBACK_HBM_GBS = 6800.0
+
+
+def parse_args():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=20)
+    p.add_argument("--warmup", type=int, default=5)
+    p.add_argument("--impl", choices=("darb", "reference"), default="darb")
+    p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--no-cpu", action="store_true")
+    return p.parse_args()
+
+
+def measured_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    except (OSError, KeyError, ValueError):
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+# ----------------------------------------------------------------------------- clocks
+class ClockSampler:
+    """nvidia-smi samples of SM clock and throttle reasons while the timed region runs."""
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.lines = []
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+            time.sleep(0.3)
+        except OSError:
+            self.proc = None
+        return self
+
+    def _read(self):
+        for ln in self.proc.stdout:
+            self.lines.append(ln.strip())
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self):
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            parts = [p.strip() for p in ln.split(",")]
+            if len(parts) < 8:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                mx.append(float(parts[1]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[4:8]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ----------------------------------------------------------------------------- distributed
+def dist_setup(args):
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        import torch
+        backend = "nccl" if torch.cuda.is_available() else "gloo"
+        if backend == "nccl":
+            torch.cuda.set_device(local)
+        dist.init_process_group(backend=backend)
+    return world, rank, local
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_over_ranks(value: float, world: int) -> float:
+    if world == 1:
+        return value
+    import torch
+    import torch.distributed as dist
+    dev = torch.device("cuda", torch.cuda.current_device()) if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([value], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+# ----------------------------------------------------------------------------- bytes
+def spmm_bytes(info, batch):
+    return (info["value_bytes"] + info["offset_bytes"] + info["meta_bytes"]
+            + info["cols"] * batch * 4 + info["rows"] * batch * 4)
+
+
+def encode_bytes(info):
+    esz = 2 if info["wtype"] == 1 else 4
+    return info["rows"] * info["cols"] * esz + info["value_bytes"] + info["offset_bytes"] + info["meta_bytes"]
+
+
+# ----------------------------------------------------------------------------- GPU arm
+class Workload:
+    """Rotating sets of device buffers for the FC6/FC7 step."""
+
+    def __init__(self, torch, darb, synth):
+        self.torch, self.darb = torch, darb
+        wl = synth.WORKLOADS[WORKLOAD]
+        dev = torch.device("cuda", torch.cuda.current_device())
+        self.dev = dev
+        self.mats = []
+        for i, (rows, cols) in enumerate(wl.shapes):
+            _, bits, m = synth.matrix(wl, i)
+            W = torch.from_numpy(bits.view(np.int16)).to(dev).view(torch.bfloat16)
+            h = darb.darb_encode(W, m)
+            exp = darb.darb_export(h)
+            info = darb.darb_info(h)
+            self.mats.append(dict(rows=rows, cols=cols, m=m, W=W, h=h, exp=exp, info=info,
+                                  bits=bits))
+        self.sets = []
+        for s in range(NSETS):
+            st = {"W": [], "enc": [], "spmm": {}, "X": {}, "Y": {}}
+            for mi, mat in enumerate(self.mats):
+                st["W"].append(mat["W"].clone())
+                val, off, _, m = mat["exp"]
+                st["enc"].append(darb.darb_import(val, off, m, darb.BF16, mat["rows"], mat["cols"]))
+                for b in BATCHES:
+                    st["spmm"][(mi, b)] = darb.darb_import(val, off, m, darb.BF16, mat["rows"], mat["cols"])
+                    X = torch.from_numpy(synth.activations(mat["cols"], b, seed=wl.seed, sub=10 * s + b)).to(dev)
+                    st["X"][(mi, b)] = X
+                    st["Y"][(mi, b)] = torch.empty((mat["rows"], b), device=dev)
+            self.sets.append(st)
+        torch.cuda.synchronize()
+        # the calls of one step, with their algorithmic bytes
+        self.calls = []
+        for mi, mat in enumerate(self.mats):
+            self.calls.append(("encode", mi, None, encode_bytes(mat["info"])))
+        for b in BATCHES:
+            for mi, mat in enumerate(self.mats):
+                self.calls.append(("spmm", mi, b, spmm_bytes(mat["info"], b)))
+        self.step_bytes = sum(c[3] for c in self.calls)
+
+    def launch(self, call, s, stream):
+        kind, mi, b, _ = call
+        st = self.sets[s % NSETS]
+        if kind == "encode":
+            self.darb.darb_reencode(st["enc"][mi], st["W"][mi], stream)
+        else:
+            self.darb.darb_spmm(st["spmm"][(mi, b)], st["X"][(mi, b)], st["Y"][(mi, b)], stream)
+
+    def check_encode(self):
+        for st in self.sets:
+            for h in st["enc"]:
+                self.darb.darb_encode_status(h)
+
+    def close(self):
+        for st in self.sets:
+            for h in st["enc"]:
+                self.darb.darb_destroy(h)
+            for h in st["spmm"].values():
+                self.darb.darb_destroy(h)
+        for mat in self.mats:
+            self.darb.darb_destroy(mat["h"])
+
+
+def run_gpu(args, world, rank, local):
+    import torch
+
+    from paper_1911_08020_gb300 import darb, synth
+    torch.cuda.set_device(local)
+    wl = Workload(torch, darb, synth)
+    stream = torch.cuda.current_stream()
+    sid = stream.cuda_stream
+    ncalls = len(wl.calls)
+
+    for s in range(args.warmup):
+        for c in wl.calls:
+            wl.launch(c, s, sid)
+    torch.cuda.synchronize()
+
+    # timed region: events around every launch give per-call device durations
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(ncalls + 1)] for _ in range(args.steps)]
+    start = torch.cuda.Event(enable_timing=True)
+    end = torch.cuda.Event(enable_timing=True)
+    barrier(world)
+    torch.cuda.synchronize()
+    with ClockSampler(local) as clk:
+        start.record(stream)
+        for s in range(args.steps):
+            ev[s][0].record(stream)
+            for i, c in enumerate(wl.calls):
+                wl.launch(c, s, sid)
+                ev[s][i + 1].record(stream)
+        end.record(stream)
+        torch.cuda.synchronize()
+    barrier(world)
+    elapsed_ms = start.elapsed_time(end)
+    wl.check_encode()
+    elapsed_ms = max_over_ranks(elapsed_ms, world)
+    ms_per_step = elapsed_ms / args.steps
+
+    per_call = np.zeros(ncalls)
+    for s in range(args.steps):
+        for i in range(ncalls):
+            per_call[i] += ev[s][i].elapsed_time(ev[s][i + 1])
+    per_call /= args.steps   # ms per launch
+    peak, peak_kind = measured_peaks()
+    parts = []
+    for i, (kind, mi, b, nbytes) in enumerate(wl.calls):
+        name = ("fc6" if mi == 0 else "fc7") + ("_encode" if kind == "encode" else f"_spmm_b{b}")
+        gbs = nbytes / (per_call[i] * 1e-3) / 1e9
+        parts.append({"call": name, "bytes": int(nbytes), "us": round(per_call[i] * 1e3, 3),
+                      "gbs": round(gbs, 1), "hbm_frac": round(gbs / peak, 4),
+                      "gflops": round(2 * wl.mats[mi]["info"]["nnzb"] * b / (per_call[i] * 1e-3) / 1e9, 1)
+                      if kind == "spmm" else None})
+    # dominant kernel: the call kind/batch with the largest share of the step
+    kinds = {}
+    for p, i in zip(parts, range(ncalls)):
+        key = p["call"].split("_", 1)[1]
+        k = kinds.setdefault(key, [0.0, 0, 0])
+        k[0] += per_call[i]
+        k[1] += p["bytes"]
+        k[2] += 1
+    dom = max(kinds, key=lambda k: kinds[k][0])
+    dom_ms, dom_bytes, dom_n = kinds[dom]
+    achieved = dom_bytes / (dom_ms * 1e-3) / 1e9
+    value = world * wl.step_bytes / (ms_per_step * 1e-3) / 1e9
+
+    result = {
+        "metric": METRIC, "value": round(value, 2), "unit": "GB/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_per_step, 5),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+        "data": "synthetic",
+        "config": {"workload": "fc6_fc7_4096x9216_4096x4096_bf16_weights",
+                   "batches": list(BATCHES), "calls_per_step": ncalls,
+                   "weights": "bf16 kept values, fp32 accumulate; X and Y fp32",
+                   "block_sizes": "per row from {16,32,64} w.p. (.4,.3,.3)",
+                   "pruning_ratio": [round(m["rows"] * m["cols"] / m["info"]["nnzb"], 2) for m in wl.mats],
+                   "l2": f"inputs rotate over {NSETS} buffer sets (>4x L2), every call reads cold HBM",
+                   "parallelism": f"replicas{world}"},
+        "roofline": {"bound": "hbm", "kernel": dom, "achieved": round(achieved, 1), "peak": peak,
+                     "peak_kind": peak_kind, "unit": "GB/s", "frac": round(achieved / peak, 4),
+                     "traffic": None},
+        "parts": parts,
+        "gpu_launches": ncalls * args.steps,
+        "clocks": clk.summary(),
+    }
+    if not args.no_e2e:
+        result["e2e"] = run_e2e(args, wl, torch, darb)
+    wl.close()
+    return result
+
+
+def run_e2e(args, wl, torch, darb):
+    """The same step through the public API from pinned host buffers."""
+    stream = torch.cuda.current_stream()
+    sid = stream.cuda_stream
+    host_W = [torch.from_numpy(m["bits"].view(np.int16)).pin_memory() for m in wl.mats]
+    host_X, host_Y = {}, {}
+    st0 = wl.sets[0]
+    for key, X in st0["X"].items():
+        host_X[key] = X.cpu().pin_memory()
+        host_Y[key] = torch.empty(st0["Y"][key].shape, dtype=torch.float32).pin_memory()
+    h2d = sum(w.numel() * 2 for w in host_W) + sum(x.numel() * 4 for x in host_X.values())
+    d2h = sum(y.numel() * 4 for y in host_Y.values())
+
+    def step(s):
+        st = wl.sets[s % NSETS]
+        for mi in range(len(wl.mats)):
+            st["W"][mi].view(torch.int16).copy_(host_W[mi], non_blocking=True)
+            darb.darb_reencode(st["enc"][mi], st["W"][mi], sid)
+        for (kind, mi, b, _) in wl.calls:
+            if kind != "spmm":
+                continue
+            key = (mi, b)
+            st["X"][key].copy_(host_X[key], non_blocking=True)
+            darb.darb_spmm(st["spmm"][key], st["X"][key], st["Y"][key], sid)
+            host_Y[key].copy_(st["Y"][key], non_blocking=True)
+
+    steps = max(3, args.steps // 2)
+    for s in range(args.warmup):
+        step(s)
+    torch.cuda.synchronize()
+    a = torch.cuda.Event(enable_timing=True)
+    b = torch.cuda.Event(enable_timing=True)
+    a.record(stream)
+    for s in range(steps):
+        step(s)
+    b.record(stream)
+    torch.cuda.synchronize()
+    ms = a.elapsed_time(b) / steps
+    return {"value": round(wl.step_bytes / (ms * 1e-3) / 1e9, 2), "unit": "GB/s",
+            "ms_per_step": round(ms, 4), "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h)}
+
+
+# ----------------------------------------------------------------------------- CPU oracle arm
+def oracle_sample(budget_s: float = 12.0):
+    """The oracle as it stands on a bounded sample of the same workload: encode of
+    FC7 and its product at batch 1 and 16.  Returns (GB/s, seconds, cores, sample)."""
+    import oracle
+    from paper_1911_08020_gb300 import synth
+    wl = synth.WORKLOADS[WORKLOAD]
+    _, bits, m = synth.matrix(wl, 1)
+    rows, cols = wl.shapes[1]
+    cores = oracle.set_threads(0)
+    X1 = synth.activations(cols, 1, seed=wl.seed, sub=91)
+    X16 = synth.activations(cols, 16, seed=wl.seed, sub=92)
+    total_bytes, total_s, reps = 0, 0.0, 0
+    while total_s < budget_s or reps == 0:
+        t0 = time.perf_counter()
+        enc = oracle.encode(bits, m, "bf16")
+        oracle.darb_spmm(enc, X1)
+        oracle.darb_spmm(enc, X16)
+        total_s += time.perf_counter() - t0
+        nnzb = int(enc.blk_ptr[-1])
+        vb = nnzb * 2
+        ob = sum(-(-cols // int(x)) * (4 if x <= 16 else 8) for x in m) // 8
+        meta = rows * 6
+        total_bytes += (rows * cols * 2 + vb + ob + meta) + sum(
+            vb + ob + meta + cols * b * 4 + rows * b * 4 for b in (1, 16))
+        reps += 1
+        if reps >= 50:
+            break
+    sample = f"FC7 4096x4096 bf16: oracle encode + darb_spmm at batch 1 and 16, x{reps}"
+    return total_bytes / total_s / 1e9, total_s, cores, sample
+
+
+def run_reference(args, world, rank):
+    if rank != 0:
+        return None
+    import oracle
+    oracle.build()
+    per_step = []
+    for s in range(args.warmup + args.steps):
+        gbs, secs, cores, sample = oracle_sample(budget_s=max(0.5, 60.0 / max(1, args.steps + args.warmup)))
+        if s >= args.warmup:
+            per_step.append(secs)
+        last = (gbs, cores, sample)
+    gbs, cores, sample = last
+    ms = 1e3 * statistics.mean(per_step)
+    return {
+        "metric": METRIC, "value": round(gbs, 3), "unit": "GB/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms, 3),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic", "impl": "reference",
+        "config": {"workload": "fc6_fc7_4096x9216_4096x4096_bf16_weights",
+                   "sample": sample, "parallelism": "cpu"},
+        "cpu_baseline": {"value": round(gbs, 3), "unit": "GB/s", "cores": cores, "kind": "oracle",
+                         "sample": sample},
+        "e2e": {"value": round(gbs, 3), "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+
+
+def main():
+    args = parse_args()
+    world, rank, local = dist_setup(args)
+    if args.impl == "reference":
+        res = run_reference(args, world, rank)
+        if rank == 0 and res is not None:
+            print(json.dumps(res), flush=True)
+        return
+    res = run_gpu(args, world, rank, local)
+    if rank == 0:
+        if not args.no_cpu and world == 1:
+            import oracle
+            oracle.build()
+            gbs, secs, cores, sample = oracle_sample()
+            res["cpu_baseline"] = {"value": round(gbs, 3), "unit": "GB/s", "cores": cores,
+                                   "kind": "oracle", "sample": sample, "seconds": round(secs, 2)}
+        print(json.dumps(res), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

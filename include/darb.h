@@ -1,0 +1,215 @@
+/*
+ * darb.h -- C ABI of libdarb: density-adaptive regular-block (DARB) pruned
+ * matrices on one GB300 GPU (sm_103a).
+ *
+ * DARB (Ren et al., "DARB: A Density-Adaptive Regular-Block Pruning for Deep
+ * Neural Networks", arXiv 1911.08020) splits every row of a weight matrix into
+ * equal blocks whose size depends on the row (Sec. 3.2), keeps the one weight of
+ * largest magnitude in each block (block-max weight masking, BMWM, Sec. 3.1),
+ * and stores per block only that value and its position inside the block
+ * (log2 m bits, Sec. 4.2).  Multiplying by such a matrix needs, per block, one
+ * small selection among m activations (Sec. 3.2, Fig. 6(b)).
+ *
+ * This library encodes dense matrices into that format on the GPU and
+ * multiplies with them, alone or fused into LSTM / GRU cell steps.
+ *
+ * Conventions shared by every call:
+ *  - Every call returns a darb_status_t and never aborts the process.
+ *  - Matrices are row-major with an explicit leading dimension in elements.
+ *    Activations X are cols x batch with the batch contiguous (row k of X
+ *    starts at X + k * ldx); outputs Y are rows x batch (row r at Y + r * ldy).
+ *  - Pointers documented as "device" must be CUDA device (or managed) memory
+ *    of the current device; "host" pointers are ordinary host memory.
+ *  - The caller owns every buffer it passes; a handle owns the encoded matrix
+ *    and any scratch it allocates, and releases both in darb_destroy.
+ *  - Work is enqueued on the caller's stream.  Only darb_encode, darb_import,
+ *    darb_export, darb_encode_status, darb_rnn_reserve and darb_destroy
+ *    synchronise; the product and step calls are asynchronous and allocate
+ *    nothing (except the RNN step scratch noted below).
+ *  - There is no CPU fallback: without a usable CUDA device the GPU calls
+ *    return DARB_ERR_CUDA.
+ */
+#ifndef DARB_H
+#define DARB_H
+
+#include <stdint.h>
+#include <cuda_runtime_api.h>
+
+#if defined(__GNUC__)
+#define DARB_API __attribute__((visibility("default")))
+#else
+#define DARB_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct darb_handle_s *darb_handle_t;
+
+typedef enum {
+    DARB_OK = 0,
+    DARB_ERR_INVALID_ARG = 1,   /* null pointer, size <= 0, ld < width, m out of [1,256],
+                                   shape mismatch, unknown or destroyed handle          */
+    DARB_ERR_NONFINITE = 2,     /* a NaN weight was found while encoding                 */
+    DARB_ERR_OOM = 3,           /* a device or host allocation failed                    */
+    DARB_ERR_CUDA = 4,          /* a CUDA runtime call or kernel launch failed           */
+    DARB_ERR_TIMEOUT = 5,       /* a bounded device-side wait gave up (reserved)         */
+    DARB_ERR_UNSUPPORTED = 6    /* arguments valid but not supported by these kernels    */
+} darb_status_t;
+
+typedef enum { DARB_F32 = 0, DARB_BF16 = 1 } darb_dtype_t;
+
+/* Largest block size the format stores (offsets take at most 8 bits). */
+#define DARB_MAX_BLOCK 256
+
+/*
+ * Density-adaptive block-size rule (Sec. 3.2, the worked example with matrix
+ * density 21.88%).  Host only; no CUDA call.
+ *   row_nnz  host int64[rows]: retained weights per row after irregular pruning,
+ *            0 <= row_nnz[r] <= cols.
+ *   m_out    host int32[rows]: block size per row.
+ * A row denser than the whole matrix has its density rounded UP to the next
+ * power-of-two density 1/m, a sparser row DOWN; m = 1 / rounded density.
+ * Readings where the paper is silent: a row exactly at the matrix density is
+ * rounded up; an empty row gets m_max; the result is clamped to [m_min, m_max].
+ * Errors: DARB_ERR_INVALID_ARG for null pointers, rows/cols <= 0, row_nnz out of
+ * range, or not 1 <= m_min <= m_max <= DARB_MAX_BLOCK.
+ */
+DARB_API darb_status_t darb_assign_block_sizes(const int64_t *row_nnz, int64_t rows, int64_t cols,
+                                      int32_t m_min, int32_t m_max, int32_t *m_out);
+
+/*
+ * BMWM encode (Sec. 3.1 steps (1)-(3), with the per-row block size of Sec. 3.2).
+ *   W      device, rows x cols, row-major, leading dimension ldw >= cols
+ *          (elements); fp32 or bf16 as wtype says.  Any alignment.
+ *   m      host int32[rows], 1 <= m[r] <= DARB_MAX_BLOCK (any value, not only
+ *          powers of two).
+ *   out    receives a new handle.
+ * Row r is split into ceil(cols / m[r]) blocks, block j covering columns
+ * [j*m[r], min((j+1)*m[r], cols)) (a shorter last block still keeps one
+ * weight).  In each block the weight of largest magnitude is kept; among
+ * equal magnitudes (including +0 / -0) the lowest column wins.  +-Inf are the
+ * largest magnitudes.  The kept value is stored bit for bit in wtype.
+ * Allocates the handle's device memory, runs on `stream` and synchronises it
+ * before returning; W may be freed afterwards.
+ * Errors: DARB_ERR_INVALID_ARG; DARB_ERR_NONFINITE if W holds a NaN (no handle
+ * is returned); DARB_ERR_OOM; DARB_ERR_CUDA.
+ */
+DARB_API darb_status_t darb_encode(const void *W, darb_dtype_t wtype, int64_t rows, int64_t cols,
+                          int64_t ldw, const int32_t *m, darb_handle_t *out, cudaStream_t stream);
+
+/*
+ * Re-run BMWM on a new W of the handle's shape and dtype, keeping its block
+ * sizes, into the handle's existing memory (e.g. after a retraining step of
+ * Sec. 4's prune-retrain loop).  Asynchronous on `stream`, allocates nothing.
+ * A NaN in W is recorded on the device and reported by darb_encode_status.
+ * The handle must not be in use by work on another stream meanwhile.
+ */
+DARB_API darb_status_t darb_reencode(darb_handle_t h, const void *W, int64_t ldw, cudaStream_t stream);
+
+/* Synchronise `stream` and report DARB_ERR_NONFINITE if the last (re)encode
+ * met a NaN, else DARB_OK.  Clears the recorded flag.                        */
+DARB_API darb_status_t darb_encode_status(darb_handle_t h, cudaStream_t stream);
+
+/*
+ * Y = W_darb X: for row r and batch column b,
+ *   Y[r, b] = sum_j val[r, j] * X[j*m_r + off[r, j], b]
+ * (block j of the row selects one activation row, Sec. 3.2 / Fig. 6(b)).
+ *   X  device fp32, cols x batch, ldx >= batch, 4-byte aligned.
+ *   Y  device fp32, rows x batch, ldy >= batch; overwritten.  Must not
+ *      overlap X.
+ * Accumulates in fp32.  Asynchronous on `stream`; allocates nothing; the
+ * handle is only read, so calls on several streams may share it.
+ * Errors: DARB_ERR_INVALID_ARG (null, batch <= 0, ld < batch); DARB_ERR_CUDA.
+ */
+DARB_API darb_status_t darb_spmm(darb_handle_t h, const float *X, int64_t ldx, int64_t batch, float *Y,
+                        int64_t ldy, cudaStream_t stream);
+
+/*
+ * One LSTM cell step whose gate matrix is the handle (rows = 4H, cols = I + H),
+ * multiplied with the stacked input [x_t; h_{t-1}].  Gate rows [0,H) = i,
+ * [H,2H) = f, [2H,3H) = g, [3H,4H) = o (the paper names LSTMs, Sec. 4.1, but
+ * writes no cell equations; this is the standard cell):
+ *   c_t = sigmoid(f) * c_{t-1} + sigmoid(i) * tanh(g),  h_t = sigmoid(o) * tanh(c_t)
+ *   x      device fp32, I x B (batch contiguous); may be NULL when I == 0
+ *   h_prev, c_prev   device fp32, H x B
+ *   bias   device fp32 [4H] added to the gate pre-activations, or NULL
+ *   h_out, c_out     device fp32, H x B; must not overlap any input
+ * Uses scratch owned by the handle (4H x B floats of gate sums and H counters),
+ * allocated by the first step call that needs more than the handle holds (that
+ * call synchronises); call darb_rnn_reserve first to size it up front.  Step
+ * calls on one handle must be ordered on one stream.
+ * Errors: DARB_ERR_INVALID_ARG (null, shape mismatch, B <= 0); DARB_ERR_OOM;
+ * DARB_ERR_CUDA.
+ */
+DARB_API darb_status_t darb_lstm_step(darb_handle_t h, int64_t I, int64_t H, int64_t B, const float *x,
+                             const float *h_prev, const float *c_prev, const float *bias,
+                             float *h_out, float *c_out, cudaStream_t stream);
+
+/*
+ * One GRU cell step whose gate matrix is the handle (rows = 3H, cols = I + H).
+ * Gate rows [0,H) = r, [H,2H) = z, [2H,3H) = n; columns [0,I) multiply x_t and
+ * [I,I+H) multiply h_{t-1}, and the two parts are kept apart (the paper names
+ * GRUs, Sec. 4.1, without equations; this is the standard cell):
+ *   a = W[:, :I] x + b_ih,  bh = W[:, I:] h + b_hh
+ *   r = sigmoid(a_r + bh_r), z = sigmoid(a_z + bh_z), n = tanh(a_n + r * bh_n)
+ *   h_t = (1 - z) * n + z * h_{t-1}
+ *   x device fp32 I x B (NULL allowed when I == 0); h_prev device fp32 H x B;
+ *   b_ih, b_hh device fp32 [3H] or NULL; h_out device fp32 H x B, not
+ *   overlapping any input.
+ * Scratch, ordering and errors as for darb_lstm_step (scratch 2 x 3H x B floats).
+ */
+DARB_API darb_status_t darb_gru_step(darb_handle_t h, int64_t I, int64_t H, int64_t B, const float *x,
+                            const float *h_prev, const float *b_ih, const float *b_hh,
+                            float *h_out, cudaStream_t stream);
+
+/* Size the handle's RNN step scratch for batches up to max_batch now, so that
+ * later step calls allocate nothing (e.g. before capturing them in a CUDA
+ * graph).  Synchronises the device.  Errors: INVALID_ARG, OOM, CUDA.          */
+DARB_API darb_status_t darb_rnn_reserve(darb_handle_t h, int64_t max_batch);
+
+typedef struct {
+    int64_t rows, cols;
+    int64_t nnzb;            /* kept weights = blocks = sum_r ceil(cols / m_r)           */
+    darb_dtype_t wtype;
+    int32_t nbins;           /* distinct block sizes                                     */
+    int32_t ngroups;         /* 32-row groups the kernels work on                        */
+    int64_t value_bytes;     /* nnzb * sizeof(value): the values the paper stores       */
+    int64_t offset_bytes;    /* stored offsets: 4 bits per block if m <= 16, else 8     */
+    int64_t meta_bytes;      /* per-row block size and pointer (int32 + uint16)         */
+    int64_t index_bits_min;  /* sum over blocks of ceil(log2 m): the paper's index bits */
+    int64_t device_bytes;    /* device memory the handle holds (incl. padding, scratch) */
+} darb_info_t;
+
+/* Shape and storage accounting of a handle (Sec. 4.2 index-storage analysis). */
+DARB_API darb_status_t darb_info(darb_handle_t h, darb_info_t *info);
+
+/*
+ * Copy the encoding out in canonical order: blocks in (row, j) order.
+ *   val      host, nnzb values of the handle's dtype (fp32 or bf16 bits)
+ *   off      host uint8[nnzb], position of the kept weight inside its block
+ *   blk_ptr  host int64[rows + 1], first block of each row; blk_ptr[rows] = nnzb
+ *   m        host int32[rows], block size of each row
+ * Any of the four may be NULL to skip it.  Synchronises the device.
+ */
+DARB_API darb_status_t darb_export(darb_handle_t h, void *val, uint8_t *off, int64_t *blk_ptr, int32_t *m);
+
+/* Build a handle from canonical host arrays (the inverse of darb_export).
+ * off[p] must be < m[r] and j*m[r] + off[p] < cols.  Synchronises `stream`.  */
+DARB_API darb_status_t darb_import(const void *val, const uint8_t *off, const int32_t *m,
+                          darb_dtype_t wtype, int64_t rows, int64_t cols, darb_handle_t *out,
+                          cudaStream_t stream);
+
+/* Release a handle and all device memory it owns; NULL is a no-op.  Waits for
+ * the device to finish using it.                                              */
+DARB_API darb_status_t darb_destroy(darb_handle_t h);
+
+/* Static, human-readable name of a status code. */
+DARB_API const char *darb_status_string(darb_status_t s);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* DARB_H */

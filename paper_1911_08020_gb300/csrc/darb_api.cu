@@ -1,0 +1,596 @@
+// darb_api.cu -- the C ABI of libdarb (include/darb.h): argument checking,
+// handle lifetime, the binned device layout, and kernel launches.
+#include "darb.h"
+#include "darb_internal.h"
+
+#include <algorithm>
+#include <cstdlib>
+#include <cstring>
+#include <mutex>
+#include <new>
+#include <numeric>
+#include <unordered_set>
+#include <vector>
+
+using darb::Format;
+using darb::Group;
+using darb::kChunk;
+using darb::kSlots;
+
+struct darb_handle_s {
+    int64_t rows = 0, cols = 0;
+    darb_dtype_t wtype = DARB_F32;
+    int64_t nnzb = 0;
+    int32_t nbins = 0;
+    // host copy of the layout
+    std::vector<Group> groups;
+    std::vector<int32_t> rowmap, rowloc, row_m;
+    int64_t val_elems = 0, off_words = 0;
+    // device memory: one allocation holding the layout, values and offsets
+    void *dmem = nullptr;
+    size_t dbytes = 0;
+    Group *d_groups = nullptr;
+    int32_t *d_rowmap = nullptr, *d_rowloc = nullptr, *d_row_m = nullptr, *d_err = nullptr;
+    void *d_vals = nullptr;
+    uint32_t *d_offs = nullptr;
+    // RNN step scratch (grown on demand)
+    float *d_gates = nullptr;
+    size_t gates_cap = 0;     // floats
+    int32_t *d_counters = nullptr;
+    size_t counters_cap = 0;  // ints
+};
+
+namespace {
+
+std::mutex g_mu;
+std::unordered_set<const darb_handle_s *> g_live;
+
+bool live(const darb_handle_s *h) {
+    std::lock_guard<std::mutex> lk(g_mu);
+    return h != nullptr && g_live.count(h) != 0;
+}
+
+// Test hook: DARB_FAIL_ALLOC=1 makes every device allocation of the library fail.
+bool alloc_fault_injected() {
+    const char *v = std::getenv("DARB_FAIL_ALLOC");
+    return v != nullptr && v[0] == '1';
+}
+
+darb_status_t dev_alloc(void **p, size_t bytes) {
+    *p = nullptr;
+    if (alloc_fault_injected()) return DARB_ERR_OOM;
+    const cudaError_t e = cudaMalloc(p, bytes);
+    if (e == cudaErrorMemoryAllocation) {
+        cudaGetLastError();
+        return DARB_ERR_OOM;
+    }
+    if (e != cudaSuccess) {
+        cudaGetLastError();
+        return DARB_ERR_CUDA;
+    }
+    return DARB_OK;
+}
+
+inline darb_status_t cuda_status(cudaError_t e) { return e == cudaSuccess ? DARB_OK : DARB_ERR_CUDA; }
+
+constexpr int64_t kMaxDim = int64_t(1) << 30;
+constexpr int64_t kMaxBatch = int64_t(1) << 19;
+
+size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
+
+int64_t ceil_div(int64_t a, int64_t b) { return (a + b - 1) / b; }
+
+// Bin rows by block size (stable: ascending m, then ascending row) and cut
+// each bin into 32-row groups.
+void build_layout(darb_handle_s *h, const int32_t *m) {
+    const int64_t rows = h->rows, cols = h->cols;
+    std::vector<int32_t> order(static_cast<size_t>(rows));
+    std::iota(order.begin(), order.end(), 0);
+    std::stable_sort(order.begin(), order.end(), [m](int32_t a, int32_t b) { return m[a] < m[b]; });
+    h->row_m.assign(m, m + rows);
+    h->rowloc.assign(static_cast<size_t>(rows), -1);
+    h->groups.clear();
+    h->rowmap.clear();
+    h->nbins = 0;
+    h->nnzb = 0;
+    int64_t val = 0, off = 0;
+    size_t i = 0;
+    while (i < order.size()) {
+        const int32_t mb = m[order[i]];
+        size_t e = i;
+        while (e < order.size() && m[order[e]] == mb) ++e;
+        ++h->nbins;
+        for (size_t s = i; s < e; s += kSlots) {
+            Group g{};
+            g.m = mb;
+            g.n = static_cast<int32_t>(ceil_div(cols, mb));
+            g.nrows = static_cast<int32_t>(std::min<size_t>(kSlots, e - s));
+            g.nib = mb <= 16 ? 1 : 0;
+            const int64_t nch = ceil_div(g.n, kChunk);
+            g.val_off = val;
+            g.off_off = off;
+            val += nch * kSlots * kChunk;
+            off += nch * kSlots * (g.nib ? 1 : 2);
+            const int32_t gi = static_cast<int32_t>(h->groups.size());
+            for (int k = 0; k < kSlots; ++k) {
+                if (k < g.nrows) {
+                    const int32_t r = order[s + k];
+                    h->rowmap.push_back(r);
+                    h->rowloc[r] = gi * kSlots + k;
+                } else {
+                    h->rowmap.push_back(-1);
+                }
+            }
+            h->nnzb += static_cast<int64_t>(g.n) * g.nrows;
+            h->groups.push_back(g);
+        }
+        i = e;
+    }
+    h->val_elems = val;
+    h->off_words = off;
+}
+
+darb_status_t alloc_device(darb_handle_s *h) {
+    const size_t esz = h->wtype == DARB_BF16 ? 2 : 4;
+    size_t o = 0;
+    const size_t o_groups = o; o = align_up(o + h->groups.size() * sizeof(Group), 256);
+    const size_t o_rowmap = o; o = align_up(o + h->rowmap.size() * 4, 256);
+    const size_t o_rowloc = o; o = align_up(o + h->rowloc.size() * 4, 256);
+    const size_t o_rowm = o;   o = align_up(o + h->row_m.size() * 4, 256);
+    const size_t o_err = o;    o = align_up(o + 4, 256);
+    const size_t o_vals = o;   o = align_up(o + static_cast<size_t>(h->val_elems) * esz, 256);
+    const size_t o_offs = o;   o = align_up(o + static_cast<size_t>(h->off_words) * 4, 256);
+    void *p = nullptr;
+    const darb_status_t st = dev_alloc(&p, o);
+    if (st != DARB_OK) return st;
+    char *b = static_cast<char *>(p);
+    h->dmem = p;
+    h->dbytes = o;
+    h->d_groups = reinterpret_cast<Group *>(b + o_groups);
+    h->d_rowmap = reinterpret_cast<int32_t *>(b + o_rowmap);
+    h->d_rowloc = reinterpret_cast<int32_t *>(b + o_rowloc);
+    h->d_row_m = reinterpret_cast<int32_t *>(b + o_rowm);
+    h->d_err = reinterpret_cast<int32_t *>(b + o_err);
+    h->d_vals = b + o_vals;
+    h->d_offs = reinterpret_cast<uint32_t *>(b + o_offs);
+    return DARB_OK;
+}
+
+darb_status_t upload_layout(darb_handle_s *h, cudaStream_t stream) {
+    cudaError_t e = cudaMemsetAsync(h->dmem, 0, h->dbytes, stream);
+    if (e == cudaSuccess)
+        e = cudaMemcpyAsync(h->d_groups, h->groups.data(), h->groups.size() * sizeof(Group),
+                            cudaMemcpyHostToDevice, stream);
+    if (e == cudaSuccess)
+        e = cudaMemcpyAsync(h->d_rowmap, h->rowmap.data(), h->rowmap.size() * 4,
+                            cudaMemcpyHostToDevice, stream);
+    if (e == cudaSuccess)
+        e = cudaMemcpyAsync(h->d_rowloc, h->rowloc.data(), h->rowloc.size() * 4,
+                            cudaMemcpyHostToDevice, stream);
+    if (e == cudaSuccess)
+        e = cudaMemcpyAsync(h->d_row_m, h->row_m.data(), h->row_m.size() * 4,
+                            cudaMemcpyHostToDevice, stream);
+    return cuda_status(e);
+}
+
+void free_handle(darb_handle_s *h) {
+    if (h == nullptr) return;
+    if (h->dmem) cudaFree(h->dmem);
+    if (h->d_gates) cudaFree(h->d_gates);
+    if (h->d_counters) cudaFree(h->d_counters);
+    delete h;
+}
+
+void register_handle(darb_handle_s *h) {
+    std::lock_guard<std::mutex> lk(g_mu);
+    g_live.insert(h);
+}
+
+Format format_of(const darb_handle_s *h) {
+    Format f{};
+    f.groups = h->d_groups;
+    f.rowmap = h->d_rowmap;
+    f.rowloc = h->d_rowloc;
+    f.row_m = h->d_row_m;
+    f.vals = h->d_vals;
+    f.offs = h->d_offs;
+    f.ngroups = static_cast<int32_t>(h->groups.size());
+    f.bf16 = h->wtype == DARB_BF16 ? 1 : 0;
+    f.rows = h->rows;
+    f.cols = h->cols;
+    return f;
+}
+
+darb::EncodeTarget target_of(darb_handle_s *h) {
+    darb::EncodeTarget t{};
+    t.groups = h->d_groups;
+    t.rowloc = h->d_rowloc;
+    t.row_m = h->d_row_m;
+    t.vals = h->d_vals;
+    t.offs = h->d_offs;
+    t.bf16 = h->wtype == DARB_BF16 ? 1 : 0;
+    t.rows = h->rows;
+    t.cols = h->cols;
+    return t;
+}
+
+bool valid_dtype(darb_dtype_t t) { return t == DARB_F32 || t == DARB_BF16; }
+
+darb_status_t check_shape_and_m(int64_t rows, int64_t cols, const int32_t *m) {
+    if (rows <= 0 || cols <= 0 || rows > kMaxDim || cols > kMaxDim || m == nullptr)
+        return DARB_ERR_INVALID_ARG;
+    for (int64_t r = 0; r < rows; ++r)
+        if (m[r] < 1 || m[r] > DARB_MAX_BLOCK) return DARB_ERR_INVALID_ARG;
+    return DARB_OK;
+}
+
+darb_status_t ensure_scratch(darb_handle_s *h, size_t gate_floats, size_t counter_ints) {
+    if (gate_floats > h->gates_cap) {
+        if (h->d_gates) {
+            cudaDeviceSynchronize();
+            cudaFree(h->d_gates);
+            h->d_gates = nullptr;
+            h->gates_cap = 0;
+        }
+        void *p = nullptr;
+        const darb_status_t st = dev_alloc(&p, gate_floats * sizeof(float));
+        if (st != DARB_OK) return st;
+        h->d_gates = static_cast<float *>(p);
+        h->gates_cap = gate_floats;
+    }
+    if (counter_ints > h->counters_cap) {
+        if (h->d_counters) {
+            cudaDeviceSynchronize();
+            cudaFree(h->d_counters);
+            h->d_counters = nullptr;
+            h->counters_cap = 0;
+        }
+        void *p = nullptr;
+        const darb_status_t st = dev_alloc(&p, counter_ints * sizeof(int32_t));
+        if (st != DARB_OK) return st;
+        if (cudaMemset(p, 0, counter_ints * sizeof(int32_t)) != cudaSuccess ||
+            cudaDeviceSynchronize() != cudaSuccess) {
+            cudaFree(p);
+            return DARB_ERR_CUDA;
+        }
+        h->d_counters = static_cast<int32_t *>(p);
+        h->counters_cap = counter_ints;
+    }
+    return DARB_OK;
+}
+
+size_t gate_floats_for(const darb_handle_s *h, int64_t B, bool gru) {
+    return static_cast<size_t>(h->rows) * static_cast<size_t>(B) * (gru ? 2 : 1);
+}
+
+size_t counter_ints_for(int64_t H, int64_t B) {
+    const int bt = darb::rnn_batch_tile(B);
+    return static_cast<size_t>(H) * static_cast<size_t>(ceil_div(B, bt));
+}
+
+bool overlaps(const void *a, size_t abytes, const void *b, size_t bbytes) {
+    if (a == nullptr || b == nullptr) return false;
+    const char *pa = static_cast<const char *>(a), *pb = static_cast<const char *>(b);
+    return pa < pb + bbytes && pb < pa + abytes;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char *darb_status_string(darb_status_t s) {
+    switch (s) {
+        case DARB_OK: return "DARB_OK";
+        case DARB_ERR_INVALID_ARG: return "DARB_ERR_INVALID_ARG";
+        case DARB_ERR_NONFINITE: return "DARB_ERR_NONFINITE";
+        case DARB_ERR_OOM: return "DARB_ERR_OOM";
+        case DARB_ERR_CUDA: return "DARB_ERR_CUDA";
+        case DARB_ERR_TIMEOUT: return "DARB_ERR_TIMEOUT";
+        case DARB_ERR_UNSUPPORTED: return "DARB_ERR_UNSUPPORTED";
+    }
+    return "DARB_ERR_UNKNOWN";
+}
+
+darb_status_t darb_assign_block_sizes(const int64_t *row_nnz, int64_t rows, int64_t cols,
+                                      int32_t m_min, int32_t m_max, int32_t *m_out) {
+    if (row_nnz == nullptr || m_out == nullptr || rows <= 0 || cols <= 0 || m_min < 1 ||
+        m_max < m_min || m_max > DARB_MAX_BLOCK)
+        return DARB_ERR_INVALID_ARG;
+    // total retained weights; a row is "dense" when nnz_r/cols >= total/(rows*cols)
+    __int128 total = 0;
+    for (int64_t r = 0; r < rows; ++r) {
+        if (row_nnz[r] < 0 || row_nnz[r] > cols) return DARB_ERR_INVALID_ARG;
+        total += row_nnz[r];
+    }
+    for (int64_t r = 0; r < rows; ++r) {
+        const int64_t nnz = row_nnz[r];
+        int64_t mm;
+        if (nnz == 0) {
+            mm = m_max;
+        } else {
+            // q = cols / nnz >= 1; dense rows take 2^floor(log2 q), sparse 2^ceil(log2 q)
+            const bool dense = static_cast<__int128>(nnz) * rows >= total;
+            int e = 0;
+            if (dense) {
+                while ((nnz << (e + 1)) <= cols) ++e;
+            } else {
+                while ((nnz << e) < cols) ++e;
+            }
+            mm = int64_t(1) << e;
+        }
+        m_out[r] = static_cast<int32_t>(std::min<int64_t>(std::max<int64_t>(mm, m_min), m_max));
+    }
+    return DARB_OK;
+}
+
+darb_status_t darb_encode(const void *W, darb_dtype_t wtype, int64_t rows, int64_t cols,
+                          int64_t ldw, const int32_t *m, darb_handle_t *out, cudaStream_t stream) {
+    if (out == nullptr) return DARB_ERR_INVALID_ARG;
+    *out = nullptr;
+    if (W == nullptr || !valid_dtype(wtype) || ldw < cols) return DARB_ERR_INVALID_ARG;
+    const size_t esz = wtype == DARB_BF16 ? 2 : 4;
+    if (reinterpret_cast<uintptr_t>(W) % esz != 0) return DARB_ERR_INVALID_ARG;
+    darb_status_t st = check_shape_and_m(rows, cols, m);
+    if (st != DARB_OK) return st;
+    darb_handle_s *h = new (std::nothrow) darb_handle_s();
+    if (h == nullptr) return DARB_ERR_OOM;
+    h->rows = rows;
+    h->cols = cols;
+    h->wtype = wtype;
+    try {
+        build_layout(h, m);
+    } catch (const std::bad_alloc &) {
+        delete h;
+        return DARB_ERR_OOM;
+    }
+    st = alloc_device(h);
+    if (st == DARB_OK) st = upload_layout(h, stream);
+    if (st == DARB_OK) st = cuda_status(darb::launch_encode(target_of(h), W, ldw, h->d_err, stream));
+    int32_t err = 0;
+    if (st == DARB_OK)
+        st = cuda_status(cudaMemcpyAsync(&err, h->d_err, 4, cudaMemcpyDeviceToHost, stream));
+    if (st == DARB_OK) st = cuda_status(cudaStreamSynchronize(stream));
+    if (st == DARB_OK && err != 0) st = DARB_ERR_NONFINITE;
+    if (st != DARB_OK) {
+        if (h->dmem) cudaStreamSynchronize(stream);
+        free_handle(h);
+        return st;
+    }
+    register_handle(h);
+    *out = h;
+    return DARB_OK;
+}
+
+darb_status_t darb_reencode(darb_handle_t h, const void *W, int64_t ldw, cudaStream_t stream) {
+    if (!live(h) || W == nullptr || ldw < h->cols) return DARB_ERR_INVALID_ARG;
+    const size_t esz = h->wtype == DARB_BF16 ? 2 : 4;
+    if (reinterpret_cast<uintptr_t>(W) % esz != 0) return DARB_ERR_INVALID_ARG;
+    return cuda_status(darb::launch_encode(target_of(h), W, ldw, h->d_err, stream));
+}
+
+darb_status_t darb_encode_status(darb_handle_t h, cudaStream_t stream) {
+    if (!live(h)) return DARB_ERR_INVALID_ARG;
+    int32_t err = 0;
+    cudaError_t e = cudaMemcpyAsync(&err, h->d_err, 4, cudaMemcpyDeviceToHost, stream);
+    if (e == cudaSuccess) e = cudaMemsetAsync(h->d_err, 0, 4, stream);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(stream);
+    if (e != cudaSuccess) return DARB_ERR_CUDA;
+    return err ? DARB_ERR_NONFINITE : DARB_OK;
+}
+
+darb_status_t darb_spmm(darb_handle_t h, const float *X, int64_t ldx, int64_t batch, float *Y,
+                        int64_t ldy, cudaStream_t stream) {
+    if (!live(h) || X == nullptr || Y == nullptr || batch <= 0 || ldx < batch || ldy < batch)
+        return DARB_ERR_INVALID_ARG;
+    if (reinterpret_cast<uintptr_t>(X) % 4 != 0 || reinterpret_cast<uintptr_t>(Y) % 4 != 0)
+        return DARB_ERR_INVALID_ARG;
+    if (batch > kMaxBatch) return DARB_ERR_UNSUPPORTED;
+    if (overlaps(X, static_cast<size_t>((h->cols - 1) * ldx + batch) * 4, Y,
+                 static_cast<size_t>((h->rows - 1) * ldy + batch) * 4))
+        return DARB_ERR_INVALID_ARG;
+    return cuda_status(darb::launch_spmm(format_of(h), X, ldx, batch, Y, ldy, stream));
+}
+
+darb_status_t darb_rnn_reserve(darb_handle_t h, int64_t max_batch) {
+    if (!live(h) || max_batch <= 0 || max_batch > kMaxBatch) return DARB_ERR_INVALID_ARG;
+    // GRU needs the larger gate buffer; the smallest tile gives the most counters
+    const int64_t units = h->rows;   // upper bound on H for either cell
+    size_t counters = 0;
+    for (int64_t b = 1; b <= std::min<int64_t>(max_batch, 8); ++b)
+        counters = std::max(counters, counter_ints_for(units, b));
+    counters = std::max(counters, counter_ints_for(units, max_batch));
+    return ensure_scratch(h, gate_floats_for(h, max_batch, true), counters);
+}
+
+static darb_status_t check_step(darb_handle_t h, int64_t I, int64_t H, int64_t B, int gates,
+                                const float *x, const float *h_prev) {
+    if (!live(h)) return DARB_ERR_INVALID_ARG;
+    if (I < 0 || H <= 0 || B <= 0 || h->rows != gates * H || h->cols != I + H)
+        return DARB_ERR_INVALID_ARG;
+    if ((I > 0 && x == nullptr) || h_prev == nullptr) return DARB_ERR_INVALID_ARG;
+    if (B > kMaxBatch) return DARB_ERR_UNSUPPORTED;
+    return DARB_OK;
+}
+
+darb_status_t darb_lstm_step(darb_handle_t h, int64_t I, int64_t H, int64_t B, const float *x,
+                             const float *h_prev, const float *c_prev, const float *bias,
+                             float *h_out, float *c_out, cudaStream_t stream) {
+    darb_status_t st = check_step(h, I, H, B, 4, x, h_prev);
+    if (st != DARB_OK) return st;
+    if (c_prev == nullptr || h_out == nullptr || c_out == nullptr) return DARB_ERR_INVALID_ARG;
+    const size_t hb = static_cast<size_t>(H * B) * 4;
+    const void *ins[4] = {x, h_prev, c_prev, bias};
+    const size_t inb[4] = {static_cast<size_t>(I * B) * 4, hb, hb, static_cast<size_t>(4 * H) * 4};
+    for (int i = 0; i < 4; ++i)
+        if (overlaps(h_out, hb, ins[i], inb[i]) || overlaps(c_out, hb, ins[i], inb[i]))
+            return DARB_ERR_INVALID_ARG;
+    if (overlaps(h_out, hb, c_out, hb)) return DARB_ERR_INVALID_ARG;
+    st = ensure_scratch(h, gate_floats_for(h, B, false), counter_ints_for(H, B));
+    if (st != DARB_OK) return st;
+    darb::RnnScratch sc{h->d_gates, h->d_counters};
+    return cuda_status(darb::launch_lstm_step(format_of(h), I, H, B, x, h_prev, c_prev, bias,
+                                              h_out, c_out, sc, stream));
+}
+
+darb_status_t darb_gru_step(darb_handle_t h, int64_t I, int64_t H, int64_t B, const float *x,
+                            const float *h_prev, const float *b_ih, const float *b_hh,
+                            float *h_out, cudaStream_t stream) {
+    darb_status_t st = check_step(h, I, H, B, 3, x, h_prev);
+    if (st != DARB_OK) return st;
+    if (h_out == nullptr) return DARB_ERR_INVALID_ARG;
+    const size_t hb = static_cast<size_t>(H * B) * 4;
+    const void *ins[4] = {x, h_prev, b_ih, b_hh};
+    const size_t inb[4] = {static_cast<size_t>(I * B) * 4, hb, static_cast<size_t>(3 * H) * 4,
+                           static_cast<size_t>(3 * H) * 4};
+    for (int i = 0; i < 4; ++i)
+        if (overlaps(h_out, hb, ins[i], inb[i])) return DARB_ERR_INVALID_ARG;
+    st = ensure_scratch(h, gate_floats_for(h, B, true), counter_ints_for(H, B));
+    if (st != DARB_OK) return st;
+    darb::RnnScratch sc{h->d_gates, h->d_counters};
+    return cuda_status(darb::launch_gru_step(format_of(h), I, H, B, x, h_prev, b_ih, b_hh, h_out,
+                                             sc, stream));
+}
+
+darb_status_t darb_info(darb_handle_t h, darb_info_t *info) {
+    if (!live(h) || info == nullptr) return DARB_ERR_INVALID_ARG;
+    darb_info_t r{};
+    r.rows = h->rows;
+    r.cols = h->cols;
+    r.nnzb = h->nnzb;
+    r.wtype = h->wtype;
+    r.nbins = h->nbins;
+    r.ngroups = static_cast<int32_t>(h->groups.size());
+    r.value_bytes = h->nnzb * (h->wtype == DARB_BF16 ? 2 : 4);
+    int64_t off_bits = 0, idx_bits = 0;
+    for (int64_t i = 0; i < h->rows; ++i) {
+        const int32_t mm = h->row_m[i];
+        const int64_t n = ceil_div(h->cols, mm);
+        off_bits += n * (mm <= 16 ? 4 : 8);
+        int b = 0;
+        while ((int64_t(1) << b) < mm) ++b;
+        idx_bits += n * b;
+    }
+    r.offset_bytes = (off_bits + 7) / 8;
+    r.meta_bytes = h->rows * 6;
+    r.index_bits_min = idx_bits;
+    r.device_bytes = static_cast<int64_t>(h->dbytes + h->gates_cap * 4 + h->counters_cap * 4);
+    *info = r;
+    return DARB_OK;
+}
+
+darb_status_t darb_export(darb_handle_t h, void *val, uint8_t *off, int64_t *blk_ptr, int32_t *m) {
+    if (!live(h)) return DARB_ERR_INVALID_ARG;
+    const size_t esz = h->wtype == DARB_BF16 ? 2 : 4;
+    std::vector<uint8_t> hv;
+    std::vector<uint32_t> ho;
+    try {
+        hv.resize(static_cast<size_t>(h->val_elems) * esz);
+        ho.resize(static_cast<size_t>(h->off_words));
+    } catch (const std::bad_alloc &) {
+        return DARB_ERR_OOM;
+    }
+    if (cudaDeviceSynchronize() != cudaSuccess) return DARB_ERR_CUDA;
+    if (cudaMemcpy(hv.data(), h->d_vals, hv.size(), cudaMemcpyDeviceToHost) != cudaSuccess ||
+        cudaMemcpy(ho.data(), h->d_offs, ho.size() * 4, cudaMemcpyDeviceToHost) != cudaSuccess)
+        return DARB_ERR_CUDA;
+    std::vector<int64_t> bp(static_cast<size_t>(h->rows) + 1, 0);
+    for (int64_t r = 0; r < h->rows; ++r) bp[r + 1] = bp[r] + ceil_div(h->cols, h->row_m[r]);
+    for (int64_t r = 0; r < h->rows; ++r) {
+        const int32_t loc = h->rowloc[r];
+        const Group &g = h->groups[loc / kSlots];
+        const int slot = loc % kSlots;
+        for (int64_t j = 0; j < g.n; ++j) {
+            const int64_t c = j / kChunk, e = j % kChunk;
+            const int64_t vi = g.val_off + (c * kSlots + slot) * kChunk + e;
+            const int64_t p = bp[r] + j;
+            if (val) std::memcpy(static_cast<char *>(val) + p * esz, hv.data() + vi * esz, esz);
+            if (off) {
+                uint32_t o;
+                if (g.nib) {
+                    o = (ho[g.off_off + c * kSlots + slot] >> (4 * e)) & 15u;
+                } else {
+                    const uint32_t w = ho[g.off_off + 2 * (c * kSlots + slot) + (e >= 4 ? 1 : 0)];
+                    o = (w >> (8 * (e & 3))) & 255u;
+                }
+                off[p] = static_cast<uint8_t>(o);
+            }
+        }
+    }
+    if (blk_ptr) std::memcpy(blk_ptr, bp.data(), bp.size() * sizeof(int64_t));
+    if (m) std::memcpy(m, h->row_m.data(), h->row_m.size() * sizeof(int32_t));
+    return DARB_OK;
+}
+
+darb_status_t darb_import(const void *val, const uint8_t *off, const int32_t *m,
+                          darb_dtype_t wtype, int64_t rows, int64_t cols, darb_handle_t *out,
+                          cudaStream_t stream) {
+    if (out == nullptr) return DARB_ERR_INVALID_ARG;
+    *out = nullptr;
+    if (val == nullptr || off == nullptr || !valid_dtype(wtype)) return DARB_ERR_INVALID_ARG;
+    darb_status_t st = check_shape_and_m(rows, cols, m);
+    if (st != DARB_OK) return st;
+    darb_handle_s *h = new (std::nothrow) darb_handle_s();
+    if (h == nullptr) return DARB_ERR_OOM;
+    h->rows = rows;
+    h->cols = cols;
+    h->wtype = wtype;
+    const size_t esz = wtype == DARB_BF16 ? 2 : 4;
+    std::vector<uint8_t> hv;
+    std::vector<uint32_t> ho;
+    try {
+        build_layout(h, m);
+        hv.assign(static_cast<size_t>(h->val_elems) * esz, 0);
+        ho.assign(static_cast<size_t>(h->off_words), 0);
+    } catch (const std::bad_alloc &) {
+        delete h;
+        return DARB_ERR_OOM;
+    }
+    int64_t p = 0;
+    for (int64_t r = 0; r < rows; ++r) {
+        const int32_t loc = h->rowloc[r];
+        const Group &g = h->groups[loc / kSlots];
+        const int slot = loc % kSlots;
+        for (int64_t j = 0; j < g.n; ++j, ++p) {
+            if (off[p] >= g.m || j * g.m + off[p] >= cols) {
+                delete h;
+                return DARB_ERR_INVALID_ARG;
+            }
+            const int64_t c = j / kChunk, e = j % kChunk;
+            const int64_t vi = g.val_off + (c * kSlots + slot) * kChunk + e;
+            std::memcpy(hv.data() + vi * esz, static_cast<const char *>(val) + p * esz, esz);
+            if (g.nib) {
+                ho[g.off_off + c * kSlots + slot] |= static_cast<uint32_t>(off[p]) << (4 * e);
+            } else {
+                ho[g.off_off + 2 * (c * kSlots + slot) + (e >= 4 ? 1 : 0)] |=
+                    static_cast<uint32_t>(off[p]) << (8 * (e & 3));
+            }
+        }
+    }
+    st = alloc_device(h);
+    if (st == DARB_OK) st = upload_layout(h, stream);
+    if (st == DARB_OK)
+        st = cuda_status(cudaMemcpyAsync(h->d_vals, hv.data(), hv.size(), cudaMemcpyHostToDevice, stream));
+    if (st == DARB_OK)
+        st = cuda_status(cudaMemcpyAsync(h->d_offs, ho.data(), ho.size() * 4, cudaMemcpyHostToDevice, stream));
+    if (st == DARB_OK) st = cuda_status(cudaStreamSynchronize(stream));
+    if (st != DARB_OK) {
+        if (h->dmem) cudaStreamSynchronize(stream);
+        free_handle(h);
+        return st;
+    }
+    register_handle(h);
+    *out = h;
+    return DARB_OK;
+}
+
+darb_status_t darb_destroy(darb_handle_t h) {
+    if (h == nullptr) return DARB_OK;
+    {
+        std::lock_guard<std::mutex> lk(g_mu);
+        if (g_live.erase(h) == 0) return DARB_ERR_INVALID_ARG;
+    }
+    free_handle(h);
+    return DARB_OK;
+}
+
+}  // extern "C"

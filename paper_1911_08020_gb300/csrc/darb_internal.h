@@ -1,0 +1,86 @@
+// darb_internal.h -- device layout of an encoded DARB matrix and the launchers
+// that the C ABI (darb_api.cu) calls.  Internal to libdarb.
+//
+// Layout in HBM (one allocation per handle):
+//
+//  * Rows are binned by block size m (Sec. 3.2 gives every row its own m) and
+//    each bin is cut into groups of 32 rows ("slots"); the last group of a bin
+//    is zero-padded.  Groups are ordered by ascending m, i.e. by descending
+//    blocks per row, so the heaviest groups are launched first.
+//  * Values of a group are stored chunk-interleaved: chunk c holds blocks
+//    [8c, 8c+8) of every slot, slot-major, 8 values per slot.  A warp whose
+//    lane i works on slot i reads a chunk with one 16-byte (bf16) or two
+//    16-byte (fp32) loads per lane, all 32 lanes contiguous.
+//  * Offsets are packed per chunk and slot into a 4-byte record of eight
+//    4-bit offsets when m <= 16, or an 8-byte record of eight 8-bit offsets
+//    otherwise (the paper's log2 m bits per index, Sec. 4.2, rounded up to a
+//    nibble or a byte so that they unpack with shifts in registers).
+//  * rowmap[g*32 + i] is the matrix row held by slot i of group g (-1: pad);
+//    rowloc[r] = g*32 + i is its inverse.
+#pragma once
+
+#include <cstdint>
+#include <cuda_runtime.h>
+
+namespace darb {
+
+constexpr int kSlots = 32;   // rows per group
+constexpr int kChunk = 8;    // blocks per chunk
+
+struct Group {
+    int32_t m;        // block size shared by the group's rows
+    int32_t n;        // blocks per row, ceil(cols / m)
+    int32_t nrows;    // slots in use (1..32)
+    int32_t nib;      // 1: 4-bit offsets (m <= 16), 0: 8-bit offsets
+    int64_t val_off;  // element index of chunk 0 / slot 0 in the value array
+    int64_t off_off;  // uint32 word index of chunk 0 / slot 0 in the offset array
+};
+
+// Everything a kernel needs to read an encoded matrix.
+struct Format {
+    const Group *groups;
+    const int32_t *rowmap;   // [ngroups * 32]
+    const int32_t *rowloc;   // [rows]
+    const int32_t *row_m;    // [rows]
+    const void *vals;        // fp32 or bf16 bit patterns
+    const uint32_t *offs;
+    int32_t ngroups;
+    int32_t bf16;            // value dtype: 0 fp32, 1 bf16
+    int64_t rows, cols;
+};
+
+// Writable view used by the encoder.
+struct EncodeTarget {
+    const Group *groups;
+    const int32_t *rowloc;
+    const int32_t *row_m;
+    void *vals;
+    uint32_t *offs;
+    int32_t bf16;
+    int64_t rows, cols;
+};
+
+// Scratch for the fused RNN steps: gate sums and per-(unit, batch tile) arrival counters.
+struct RnnScratch {
+    float *gates;      // rows x B (LSTM) or 2 x rows x B (GRU: x part then h part)
+    int32_t *counters; // units x batch tiles, zero between launches
+};
+
+cudaError_t launch_encode(const EncodeTarget &t, const void *W, int64_t ldw, int32_t *err_flag,
+                          cudaStream_t stream);
+
+cudaError_t launch_spmm(const Format &f, const float *X, int64_t ldx, int64_t batch, float *Y,
+                        int64_t ldy, cudaStream_t stream);
+
+cudaError_t launch_lstm_step(const Format &f, int64_t I, int64_t H, int64_t B, const float *x,
+                             const float *h_prev, const float *c_prev, const float *bias,
+                             float *h_out, float *c_out, RnnScratch s, cudaStream_t stream);
+
+cudaError_t launch_gru_step(const Format &f, int64_t I, int64_t H, int64_t B, const float *x,
+                            const float *h_prev, const float *b_ih, const float *b_hh,
+                            float *h_out, RnnScratch s, cudaStream_t stream);
+
+// Batch-tile width the RNN step kernels use for a batch of B (sizes the counters).
+int rnn_batch_tile(int64_t B);
+
+}  // namespace darb
