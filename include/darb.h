@@ -23,7 +23,7 @@
  *  - The caller owns every buffer it passes; a handle owns the encoded matrix
  *    and any scratch it allocates, and releases both in darb_destroy.
  *  - Work is enqueued on the caller's stream.  Only darb_encode, darb_import,
- *    darb_export, darb_encode_status, darb_rnn_reserve and darb_destroy
+ *    darb_export, darb_sync_status, darb_rnn_reserve and darb_destroy
  *    synchronise; the product and step calls are asynchronous and allocate
  *    nothing (except the RNN step scratch noted below).
  *  - There is no CPU fallback: without a usable CUDA device the GPU calls
@@ -103,14 +103,16 @@ DARB_API darb_status_t darb_encode(const void *W, darb_dtype_t wtype, int64_t ro
  * Re-run BMWM on a new W of the handle's shape and dtype, keeping its block
  * sizes, into the handle's existing memory (e.g. after a retraining step of
  * Sec. 4's prune-retrain loop).  Asynchronous on `stream`, allocates nothing.
- * A NaN in W is recorded on the device and reported by darb_encode_status.
+ * A NaN in W is recorded on the device and reported by darb_sync_status.
  * The handle must not be in use by work on another stream meanwhile.
  */
 DARB_API darb_status_t darb_reencode(darb_handle_t h, const void *W, int64_t ldw, cudaStream_t stream);
 
-/* Synchronise `stream` and report DARB_ERR_NONFINITE if the last (re)encode
- * met a NaN, else DARB_OK.  Clears the recorded flag.                        */
-DARB_API darb_status_t darb_encode_status(darb_handle_t h, cudaStream_t stream);
+/* Synchronise `stream` and report what the handle's kernels recorded on the
+ * device since the last call, then clear it: DARB_ERR_TIMEOUT if a bounded
+ * wait for a bulk copy gave up (results of that call are not valid), else
+ * DARB_ERR_NONFINITE if a (re)encode met a NaN, else DARB_OK.                */
+DARB_API darb_status_t darb_sync_status(darb_handle_t h, cudaStream_t stream);
 
 /*
  * Y = W_darb X: for row r and batch column b,

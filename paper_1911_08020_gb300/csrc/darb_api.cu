@@ -2,6 +2,7 @@
 // handle lifetime, the binned device layout, and kernel launches.
 #include "darb.h"
 #include "darb_internal.h"
+#include "tma.cuh"
 
 #include <algorithm>
 #include <cstdlib>
@@ -25,14 +26,21 @@ struct darb_handle_s {
     // host copy of the layout
     std::vector<Group> groups;
     std::vector<int32_t> rowmap, rowloc, row_m;
+    std::vector<int2> enc_tiles;   // (row, first block) of every encoder tile
     int64_t val_elems = 0, off_words = 0;
     // device memory: one allocation holding the layout, values and offsets
     void *dmem = nullptr;
     size_t dbytes = 0;
     Group *d_groups = nullptr;
-    int32_t *d_rowmap = nullptr, *d_rowloc = nullptr, *d_row_m = nullptr, *d_err = nullptr;
+    int2 *d_tiles = nullptr;
+    int32_t *d_rowmap = nullptr, *d_rowloc = nullptr, *d_row_m = nullptr, *d_status = nullptr;
     void *d_vals = nullptr;
     uint32_t *d_offs = nullptr;
+    // PDL prefetch of the handle's data is safe only once no re-encode of it can
+    // still be running: reencode_event marks the last one; in_graph disables it
+    cudaEvent_t reencode_event = nullptr;
+    bool reencode_pending = false;
+    bool reencoded_in_graph = false;
     // RNN step scratch (grown on demand)
     float *d_gates = nullptr;
     size_t gates_cap = 0;     // floats
@@ -128,12 +136,20 @@ void build_layout(darb_handle_s *h, const int32_t *m) {
     }
     h->val_elems = val;
     h->off_words = off;
+    h->enc_tiles.clear();
+    for (int64_t r = 0; r < rows; ++r) {
+        const int tb = darb::enc_tile_blocks(m[r]);
+        const int64_t n = ceil_div(cols, m[r]);
+        for (int64_t jt = 0; jt < n; jt += tb)
+            h->enc_tiles.push_back(make_int2(static_cast<int>(r), static_cast<int>(jt)));
+    }
 }
 
 darb_status_t alloc_device(darb_handle_s *h) {
     const size_t esz = h->wtype == DARB_BF16 ? 2 : 4;
     size_t o = 0;
     const size_t o_groups = o; o = align_up(o + h->groups.size() * sizeof(Group), 256);
+    const size_t o_tiles = o;  o = align_up(o + h->enc_tiles.size() * sizeof(int2), 256);
     const size_t o_rowmap = o; o = align_up(o + h->rowmap.size() * 4, 256);
     const size_t o_rowloc = o; o = align_up(o + h->rowloc.size() * 4, 256);
     const size_t o_rowm = o;   o = align_up(o + h->row_m.size() * 4, 256);
@@ -147,10 +163,11 @@ darb_status_t alloc_device(darb_handle_s *h) {
     h->dmem = p;
     h->dbytes = o;
     h->d_groups = reinterpret_cast<Group *>(b + o_groups);
+    h->d_tiles = reinterpret_cast<int2 *>(b + o_tiles);
     h->d_rowmap = reinterpret_cast<int32_t *>(b + o_rowmap);
     h->d_rowloc = reinterpret_cast<int32_t *>(b + o_rowloc);
     h->d_row_m = reinterpret_cast<int32_t *>(b + o_rowm);
-    h->d_err = reinterpret_cast<int32_t *>(b + o_err);
+    h->d_status = reinterpret_cast<int32_t *>(b + o_err);
     h->d_vals = b + o_vals;
     h->d_offs = reinterpret_cast<uint32_t *>(b + o_offs);
     return DARB_OK;
@@ -160,6 +177,9 @@ darb_status_t upload_layout(darb_handle_s *h, cudaStream_t stream) {
     cudaError_t e = cudaMemsetAsync(h->dmem, 0, h->dbytes, stream);
     if (e == cudaSuccess)
         e = cudaMemcpyAsync(h->d_groups, h->groups.data(), h->groups.size() * sizeof(Group),
+                            cudaMemcpyHostToDevice, stream);
+    if (e == cudaSuccess)
+        e = cudaMemcpyAsync(h->d_tiles, h->enc_tiles.data(), h->enc_tiles.size() * sizeof(int2),
                             cudaMemcpyHostToDevice, stream);
     if (e == cudaSuccess)
         e = cudaMemcpyAsync(h->d_rowmap, h->rowmap.data(), h->rowmap.size() * 4,
@@ -178,6 +198,7 @@ void free_handle(darb_handle_s *h) {
     if (h->dmem) cudaFree(h->dmem);
     if (h->d_gates) cudaFree(h->d_gates);
     if (h->d_counters) cudaFree(h->d_counters);
+    if (h->reencode_event) cudaEventDestroy(h->reencode_event);
     delete h;
 }
 
@@ -194,6 +215,7 @@ Format format_of(const darb_handle_s *h) {
     f.row_m = h->d_row_m;
     f.vals = h->d_vals;
     f.offs = h->d_offs;
+    f.status = h->d_status;
     f.ngroups = static_cast<int32_t>(h->groups.size());
     f.bf16 = h->wtype == DARB_BF16 ? 1 : 0;
     f.rows = h->rows;
@@ -206,6 +228,8 @@ darb::EncodeTarget target_of(darb_handle_s *h) {
     t.groups = h->d_groups;
     t.rowloc = h->d_rowloc;
     t.row_m = h->d_row_m;
+    t.tiles = h->d_tiles;
+    t.ntiles = static_cast<int32_t>(h->enc_tiles.size());
     t.vals = h->d_vals;
     t.offs = h->d_offs;
     t.bf16 = h->wtype == DARB_BF16 ? 1 : 0;
@@ -257,6 +281,25 @@ darb_status_t ensure_scratch(darb_handle_s *h, size_t gate_floats, size_t counte
         h->counters_cap = counter_ints;
     }
     return DARB_OK;
+}
+
+// May a kernel read the handle's values before the previous kernel on `stream`
+// has finished?  Yes unless a re-encode of this handle might still be running.
+bool early_ok(darb_handle_s *h, cudaStream_t stream) {
+    if (h->reencoded_in_graph) return false;
+    if (!h->reencode_pending) return true;
+    cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+    if (cudaStreamIsCapturing(stream, &cs) != cudaSuccess || cs != cudaStreamCaptureStatusNone) {
+        cudaGetLastError();
+        return false;
+    }
+    const cudaError_t q = cudaEventQuery(h->reencode_event);
+    if (q == cudaSuccess) {
+        h->reencode_pending = false;
+        return true;
+    }
+    cudaGetLastError();
+    return false;
 }
 
 size_t gate_floats_for(const darb_handle_s *h, int64_t B, bool gru) {
@@ -345,10 +388,10 @@ darb_status_t darb_encode(const void *W, darb_dtype_t wtype, int64_t rows, int64
     }
     st = alloc_device(h);
     if (st == DARB_OK) st = upload_layout(h, stream);
-    if (st == DARB_OK) st = cuda_status(darb::launch_encode(target_of(h), W, ldw, h->d_err, stream));
+    if (st == DARB_OK) st = cuda_status(darb::launch_encode(target_of(h), W, ldw, h->d_status, stream));
     int32_t err = 0;
     if (st == DARB_OK)
-        st = cuda_status(cudaMemcpyAsync(&err, h->d_err, 4, cudaMemcpyDeviceToHost, stream));
+        st = cuda_status(cudaMemcpyAsync(&err, h->d_status, 4, cudaMemcpyDeviceToHost, stream));
     if (st == DARB_OK) st = cuda_status(cudaStreamSynchronize(stream));
     if (st == DARB_OK && err != 0) st = DARB_ERR_NONFINITE;
     if (st != DARB_OK) {
@@ -365,17 +408,31 @@ darb_status_t darb_reencode(darb_handle_t h, const void *W, int64_t ldw, cudaStr
     if (!live(h) || W == nullptr || ldw < h->cols) return DARB_ERR_INVALID_ARG;
     const size_t esz = h->wtype == DARB_BF16 ? 2 : 4;
     if (reinterpret_cast<uintptr_t>(W) % esz != 0) return DARB_ERR_INVALID_ARG;
-    return cuda_status(darb::launch_encode(target_of(h), W, ldw, h->d_err, stream));
+    darb_status_t st = cuda_status(darb::launch_encode(target_of(h), W, ldw, h->d_status, stream));
+    if (st != DARB_OK) return st;
+    cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+    if (cudaStreamIsCapturing(stream, &cs) != cudaSuccess || cs != cudaStreamCaptureStatusNone) {
+        cudaGetLastError();
+        h->reencoded_in_graph = true;
+        return DARB_OK;
+    }
+    if (h->reencode_event == nullptr &&
+        cudaEventCreateWithFlags(&h->reencode_event, cudaEventDisableTiming) != cudaSuccess)
+        return DARB_ERR_CUDA;
+    if (cudaEventRecord(h->reencode_event, stream) != cudaSuccess) return DARB_ERR_CUDA;
+    h->reencode_pending = true;
+    return DARB_OK;
 }
 
-darb_status_t darb_encode_status(darb_handle_t h, cudaStream_t stream) {
+darb_status_t darb_sync_status(darb_handle_t h, cudaStream_t stream) {
     if (!live(h)) return DARB_ERR_INVALID_ARG;
-    int32_t err = 0;
-    cudaError_t e = cudaMemcpyAsync(&err, h->d_err, 4, cudaMemcpyDeviceToHost, stream);
-    if (e == cudaSuccess) e = cudaMemsetAsync(h->d_err, 0, 4, stream);
+    int32_t bits = 0;
+    cudaError_t e = cudaMemcpyAsync(&bits, h->d_status, 4, cudaMemcpyDeviceToHost, stream);
+    if (e == cudaSuccess) e = cudaMemsetAsync(h->d_status, 0, 4, stream);
     if (e == cudaSuccess) e = cudaStreamSynchronize(stream);
     if (e != cudaSuccess) return DARB_ERR_CUDA;
-    return err ? DARB_ERR_NONFINITE : DARB_OK;
+    if (bits & darb::kStatusTimeout) return DARB_ERR_TIMEOUT;
+    return (bits & darb::kStatusNaN) ? DARB_ERR_NONFINITE : DARB_OK;
 }
 
 darb_status_t darb_spmm(darb_handle_t h, const float *X, int64_t ldx, int64_t batch, float *Y,
@@ -388,7 +445,8 @@ darb_status_t darb_spmm(darb_handle_t h, const float *X, int64_t ldx, int64_t ba
     if (overlaps(X, static_cast<size_t>((h->cols - 1) * ldx + batch) * 4, Y,
                  static_cast<size_t>((h->rows - 1) * ldy + batch) * 4))
         return DARB_ERR_INVALID_ARG;
-    return cuda_status(darb::launch_spmm(format_of(h), X, ldx, batch, Y, ldy, stream));
+    return cuda_status(
+        darb::launch_spmm(format_of(h), X, ldx, batch, Y, ldy, early_ok(h, stream), stream));
 }
 
 darb_status_t darb_rnn_reserve(darb_handle_t h, int64_t max_batch) {

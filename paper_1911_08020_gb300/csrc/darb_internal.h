@@ -26,6 +26,11 @@ namespace darb {
 
 constexpr int kSlots = 32;   // rows per group
 constexpr int kChunk = 8;    // blocks per chunk
+constexpr int kEncTileElems = 12288;   // columns of W the encoder stages per tile, at most
+
+// Blocks of a row with block size m that one encoder tile covers: whole
+// blocks, a multiple of the chunk so that offset records never straddle tiles.
+inline __host__ __device__ int enc_tile_blocks(int m) { return (kEncTileElems / m) / kChunk * kChunk; }
 
 struct Group {
     int32_t m;        // block size shared by the group's rows
@@ -44,6 +49,7 @@ struct Format {
     const int32_t *row_m;    // [rows]
     const void *vals;        // fp32 or bf16 bit patterns
     const uint32_t *offs;
+    int32_t *status;         // sticky device status bits (NaN seen, wait timed out)
     int32_t ngroups;
     int32_t bf16;            // value dtype: 0 fp32, 1 bf16
     int64_t rows, cols;
@@ -54,6 +60,8 @@ struct EncodeTarget {
     const Group *groups;
     const int32_t *rowloc;
     const int32_t *row_m;
+    const int2 *tiles;       // (row, first block) of every encoder tile, row-major
+    int32_t ntiles;
     void *vals;
     uint32_t *offs;
     int32_t bf16;
@@ -66,11 +74,13 @@ struct RnnScratch {
     int32_t *counters; // units x batch tiles, zero between launches
 };
 
-cudaError_t launch_encode(const EncodeTarget &t, const void *W, int64_t ldw, int32_t *err_flag,
+cudaError_t launch_encode(const EncodeTarget &t, const void *W, int64_t ldw, int32_t *status,
                           cudaStream_t stream);
 
+// `early`: the handle's data is known to be complete, so a kernel may start
+// reading it before the previous kernel on the stream has finished (PDL).
 cudaError_t launch_spmm(const Format &f, const float *X, int64_t ldx, int64_t batch, float *Y,
-                        int64_t ldy, cudaStream_t stream);
+                        int64_t ldy, bool early, cudaStream_t stream);
 
 cudaError_t launch_lstm_step(const Format &f, int64_t I, int64_t H, int64_t B, const float *x,
                              const float *h_prev, const float *c_prev, const float *bias,
@@ -82,5 +92,8 @@ cudaError_t launch_gru_step(const Format &f, int64_t I, int64_t H, int64_t B, co
 
 // Batch-tile width the RNN step kernels use for a batch of B (sizes the counters).
 int rnn_batch_tile(int64_t B);
+
+// Streaming multiprocessors of the current device (cached).
+int sm_count();
 
 }  // namespace darb

@@ -4,190 +4,220 @@
 // into blocks of m_r columns, keep the weight of largest magnitude in each
 // block (lowest column on a tie), store its value and its offset in the block.
 //
-// One CTA per matrix row.  The CTA streams the row (or a tile of whole blocks
-// of it) from HBM into shared memory with 16-byte loads, widening bf16 to fp32
-// (exact), and flags NaNs on the way.  Then each thread scans one block.  Blocks
-// are m words apart, so a straight scan would make lanes collide on shared
-// memory banks whenever m is even; each lane instead starts its scan at a
-// rotated position s(lane) = (lane * 2^a) / 32, a = min(v2(m), 5), and wraps
-// around.  Lanes that share a bank offset t*m mod 32 then start 1..2^a-1 words
-// apart, which makes every scan step conflict-free for any m.  Because the scan
-// order is rotated, a tie is resolved explicitly by the smaller offset.
+// The work is a list of tiles (a row, or a run of whole blocks of a long row).
+// A persistent grid (two or three CTAs per SM) walks the list; each CTA keeps
+// the bulk (TMA) copies of its next tiles in flight in a ring of shared-memory
+// buffers while it scans the current one, so the HBM read of W -- the only
+// large traffic -- streams without stalls.  Tiles are scanned where the copy
+// put them; positions past the row's end are zero-filled, which can never beat
+// a real element of the block (it comes later, and ties go to the lowest
+// column).  A NaN anywhere in a block would be that block's largest magnitude,
+// so checking each block's winner finds every NaN at no extra cost.
 //
-// The kernel is bound by the HBM read of W: it reads rows*cols elements once
-// and writes one value and 4-8 bits per block.
+// Scan: each thread takes one block.  Blocks are m words apart, so a straight
+// scan makes lanes collide on shared-memory banks whenever m is even; each lane
+// instead starts at a rotated position s(lane) = (lane * 2^a) / 32,
+// a = min(v2(m), 5), and wraps around.  Lanes that share a bank offset
+// t*m mod 32 then start 1..2^a-1 words apart, so every scan step is
+// conflict-free for any m.  Because the order is rotated, ties are resolved
+// explicitly by the smaller offset: for bf16, key = |w| << 16 | (0xFFFF - offset)
+// and one unsigned max per element does both; fp32 compares (|w|, offset).
 #include "darb_internal.h"
+#include "launch.cuh"
+#include "tma.cuh"
 
-#include <cuda_bf16.h>
+#include <algorithm>
+#include <type_traits>
 
 namespace darb {
 namespace {
 
 constexpr int kEncThreads = 256;
-constexpr int kEncTileElems = 12288;   // 48 KB of fp32 staging per CTA
 
 template <bool BF16>
-__device__ __forceinline__ float load_w(const void *row, int64_t c) {
-    if constexpr (BF16) {
-        uint32_t b = static_cast<const uint16_t *>(row)[c];
-        return __uint_as_float(b << 16);
-    } else {
-        return static_cast<const float *>(row)[c];
-    }
+__host__ __device__ constexpr int raw_bytes() { return kEncTileElems * (BF16 ? 2 : 4) + 128; }
+
+template <bool BF16>
+__host__ __device__ constexpr int enc_stages() { return BF16 ? 3 : 2; }
+
+template <bool BF16>
+__host__ __device__ constexpr size_t encode_smem() {
+    return 128 + size_t(enc_stages<BF16>()) * raw_bytes<BF16>();
 }
 
-// Stage columns [c0, c1) of one row into smem (as fp32); returns true if a NaN was seen.
+struct TileGeo {
+    int64_t r;
+    int jt, nb, m, span;     // first block, blocks, block size, columns
+    const char *gaddr;       // first byte of the tile in W
+    int off0;                // gaddr - (gaddr rounded down to 16 bytes)
+    int blo, bhi;            // bulk-copied byte range, relative to the rounded-down address
+};
+
 template <bool BF16>
-__device__ __forceinline__ bool stage_row(const void *row, int64_t c0, int64_t c1, float *tile) {
-    bool nan = false;
-    const int tid = threadIdx.x;
+__device__ __forceinline__ TileGeo tile_geo(const EncodeTarget &t, const void *W, int64_t ldw, int i) {
     constexpr int kEsz = BF16 ? 2 : 4;
-    constexpr int kPerVec = 16 / kEsz;
-    const char *base = static_cast<const char *>(row);
-    // head: up to the first 16-byte aligned column
-    int64_t a0 = c0;
-    uintptr_t addr0 = reinterpret_cast<uintptr_t>(base + c0 * kEsz);
-    int64_t mis = (addr0 & 15) ? (16 - (addr0 & 15)) / kEsz : 0;
-    if ((addr0 & (kEsz - 1)) != 0) mis = c1 - c0;   // not even element-aligned for vectors
-    int64_t head_end = min(c1, a0 + mis);
-    for (int64_t c = c0 + tid; c < head_end; c += kEncThreads) {
-        float v = load_w<BF16>(row, c);
-        nan |= isnan(v);
-        tile[c - c0] = v;
-    }
-    int64_t nvec = (c1 - head_end) / kPerVec;
-    const uint4 *vp = reinterpret_cast<const uint4 *>(base + head_end * kEsz);
-    for (int64_t i = tid; i < nvec; i += kEncThreads) {
-        uint4 q = __ldcs(vp + i);   // streamed once: evict-first
-        uint32_t w[4] = {q.x, q.y, q.z, q.w};
-        float *dst = tile + (head_end - c0) + i * kPerVec;
-        if constexpr (BF16) {
-#pragma unroll
-            for (int e = 0; e < 4; ++e) {
-                float lo = __uint_as_float(w[e] << 16);
-                float hi = __uint_as_float(w[e] & 0xFFFF0000u);
-                nan |= isnan(lo) | isnan(hi);
-                dst[2 * e] = lo;
-                dst[2 * e + 1] = hi;
-            }
-        } else {
-#pragma unroll
-            for (int e = 0; e < 4; ++e) {
-                float v = __uint_as_float(w[e]);
-                nan |= isnan(v);
-                dst[e] = v;
-            }
-        }
-    }
-    for (int64_t c = head_end + nvec * kPerVec + tid; c < c1; c += kEncThreads) {
-        float v = load_w<BF16>(row, c);
-        nan |= isnan(v);
-        tile[c - c0] = v;
-    }
-    return nan;
+    TileGeo g;
+    const int2 tl = t.tiles[i];
+    g.r = tl.x;
+    g.jt = tl.y;
+    g.m = t.row_m[g.r];
+    const int n = t.groups[t.rowloc[g.r] / kSlots].n;
+    g.nb = min(enc_tile_blocks(g.m), n - g.jt);
+    const int64_t c0 = int64_t(g.jt) * g.m;
+    const int64_t c1 = min(t.cols, c0 + int64_t(g.nb) * g.m);
+    g.span = static_cast<int>(c1 - c0);
+    g.gaddr = static_cast<const char *>(W) + (g.r * ldw + c0) * kEsz;
+    const uintptr_t a = reinterpret_cast<uintptr_t>(g.gaddr);
+    g.off0 = static_cast<int>(a & 15);
+    g.blo = (g.off0 + 15) & ~15;
+    g.bhi = (g.off0 + g.span * kEsz) & ~15;
+    if (g.bhi < g.blo) g.bhi = g.blo;
+    return g;
 }
 
 template <bool BF16>
 __global__ void __launch_bounds__(kEncThreads)
-encode_kernel(EncodeTarget t, const void *W, int64_t ldw, int32_t *err_flag) {
-    __shared__ float tile[kEncTileElems];
-    const int64_t r = blockIdx.x;
-    const int m = t.row_m[r];
-    const int loc = t.rowloc[r];
-    const Group grp = t.groups[loc / kSlots];
-    const int slot = loc % kSlots;
-    const int n = grp.n;
-    const int64_t cols = t.cols;
-    const int lane = threadIdx.x & 31;
-    const char *row = static_cast<const char *>(W) + r * ldw * (BF16 ? 2 : 4);
+encode_kernel(EncodeTarget t, const void *W, int64_t ldw, int32_t *status) {
+    constexpr int kEsz = BF16 ? 2 : 4;
+    constexpr int kStages = enc_stages<BF16>();
+    using elem_t = typename std::conditional<BF16, uint16_t, uint32_t>::type;
+    extern __shared__ __align__(128) unsigned char sm[];
+    uint64_t *bar = reinterpret_cast<uint64_t *>(sm);   // one per stage
+    unsigned char *const raw0 = sm + 128;               // stage s at raw0 + s * raw_bytes
+    const int tid = threadIdx.x, lane = tid & 31;
 
-    // blocks per tile: whole blocks, a multiple of the chunk so offset records
-    // never straddle two tiles
-    const int tb = (kEncTileElems / m) / kChunk * kChunk;
-    // rotation that makes the per-thread scans bank-conflict-free
-    const int a = min(__ffs(m) - 1, 5);
-    const int rot = (lane << a) >> 5;
+    pdl_launch_dependents();
+    if (tid == 0) {
+        for (int s = 0; s < kStages; ++s) mbar_init(&bar[s], 1);
+        fence_mbar_init();
+    }
+    __syncthreads();
+    pdl_wait_previous();   // W may come from the previous kernel; outputs may still be read by it
 
-    bool nan = false;
-    for (int jt = 0; jt < n; jt += tb) {
-        const int nb = min(tb, n - jt);
-        const int64_t c0 = static_cast<int64_t>(jt) * m;
-        const int64_t c1 = min(cols, c0 + static_cast<int64_t>(nb) * m);
-        __syncthreads();   // previous tile fully consumed
-        nan |= stage_row<BF16>(row, c0, c1, tile);
+    auto issue = [&](int i, int s) {
+        const TileGeo g = tile_geo<BF16>(t, W, ldw, i);
+        const uint32_t bytes = uint32_t(g.bhi - g.blo);
+        mbar_arrive_expect_tx(&bar[s], bytes);
+        if (bytes > 0) bulk_g2s(raw0 + s * raw_bytes<BF16>() + g.blo, g.gaddr - g.off0 + g.blo, bytes, &bar[s]);
+    };
+
+    bool nan = false, ok = true;
+    uint32_t phases = 0u;   // bit s: parity of stage s's next phase
+    int it = 0;
+    if (tid == 0)
+        for (int k = 0; k < kStages - 1; ++k) {
+            const int i = blockIdx.x + k * gridDim.x;
+            if (i < t.ntiles) issue(i, k);
+        }
+    for (int i = blockIdx.x; i < t.ntiles; i += gridDim.x, ++it) {
+        const int s = it % kStages;
+        const TileGeo g = tile_geo<BF16>(t, W, ldw, i);
+        const int iahead = i + (kStages - 1) * gridDim.x;
+        if (iahead < t.ntiles && tid == 0) {
+            fence_proxy_async_smem();   // earlier generic accesses to that stage come first
+            issue(iahead, (it + kStages - 1) % kStages);
+        }
+        ok = __syncthreads_and(mbar_wait(&bar[s], (phases >> s) & 1u));
+        phases ^= 1u << s;
+        if (!ok) break;
+        const int m = g.m;
+        const int padded = g.nb * m;   // <= kEncTileElems
+        // element c of the tile sits at word c of `e`; fill the bytes the bulk
+        // copy did not cover (unaligned head and tail) and zero the padding
+        elem_t *e = reinterpret_cast<elem_t *>(raw0 + s * raw_bytes<BF16>() + g.off0);
+        const elem_t *src = reinterpret_cast<const elem_t *>(g.gaddr);
+        const int ehead = (g.blo - g.off0) / kEsz, etail = (g.bhi - g.off0) / kEsz;
+        for (int c = tid; c < ehead && c < padded; c += kEncThreads) e[c] = c < g.span ? __ldg(src + c) : elem_t(0);
+        for (int c = etail + tid; c < padded; c += kEncThreads) e[c] = c < g.span ? __ldg(src + c) : elem_t(0);
         __syncthreads();
-        const int span = static_cast<int>(c1 - c0);
-        // uniform trip count so every lane reaches the shuffles below
-        for (int base = 0; base < nb; base += kEncThreads) {
-            const int jj = base + threadIdx.x;
-            const int j = jt + jj;
+        // ---- one block per thread
+        const int loc = t.rowloc[g.r];
+        const Group grp = t.groups[loc / kSlots];
+        const int slot = loc % kSlots;
+        const int a = min(__ffs(m) - 1, 5);
+        const int rot = (lane << a) >> 5;
+        for (int base = 0; base < g.nb; base += kEncThreads) {
+            const int jj = base + tid;
+            const int j = g.jt + jj;
             uint32_t best_o = 0;
-            if (jj < nb) {
-                const int lo = jj * m;
-                const int len = min(m, span - lo);
-                uint32_t best_a = 0;
-                best_o = m;   // sentinel: any element (|w| >= 0) replaces it
-                int o = rot >= m ? rot % m : rot;
-                for (int k = 0; k < m; ++k) {
-                    if (o < len) {
-                        const uint32_t av = __float_as_uint(tile[lo + o]) & 0x7FFFFFFFu;
-                        if (av > best_a || (av == best_a && static_cast<uint32_t>(o) < best_o)) {
-                            best_a = av;
-                            best_o = o;
-                        }
-                    }
-                    o = (o + 1 == m) ? 0 : o + 1;
-                }
-                const float kept = tile[lo + best_o];
-                const int64_t vi = grp.val_off +
-                                   (static_cast<int64_t>(j / kChunk) * kSlots + slot) * kChunk +
-                                   (j % kChunk);
+            if (jj < g.nb) {
+                const elem_t *blk = e + jj * m;
+                int o = rot;
                 if constexpr (BF16) {
-                    static_cast<uint16_t *>(t.vals)[vi] =
-                        static_cast<uint16_t>(__float_as_uint(kept) >> 16);
+                    uint32_t best = 0;
+                    for (int k = 0; k < m; ++k) {
+                        best = max(best, ((uint32_t(blk[o]) & 0x7FFFu) << 16) | (0xFFFFu - uint32_t(o)));
+                        o = (o + 1 == m) ? 0 : o + 1;
+                    }
+                    best_o = 0xFFFFu - (best & 0xFFFFu);
+                    nan |= (best >> 16) > 0x7F80u;
                 } else {
-                    static_cast<float *>(t.vals)[vi] = kept;
+                    uint32_t best_a = 0;
+                    best_o = uint32_t(m);
+                    for (int k = 0; k < m; ++k) {
+                        const uint32_t av = blk[o] & 0x7FFFFFFFu;
+                        if (av > best_a || (av == best_a && uint32_t(o) < best_o)) {
+                            best_a = av;
+                            best_o = uint32_t(o);
+                        }
+                        o = (o + 1 == m) ? 0 : o + 1;
+                    }
+                    nan |= best_a > 0x7F800000u;
                 }
+                const int64_t vi = grp.val_off + (int64_t(j / kChunk) * kSlots + slot) * kChunk + (j % kChunk);
+                static_cast<elem_t *>(t.vals)[vi] = blk[best_o];
             }
             // pack the 8 offsets of a chunk: lanes 8q..8q+7 hold blocks 8c..8c+7
-            const int e = j % kChunk;
+            const int q = j % kChunk;
             uint32_t lo_w, hi_w;
             if (grp.nib) {
-                lo_w = (jj < nb) ? (best_o << (4 * e)) : 0u;
+                lo_w = (jj < g.nb) ? (best_o << (4 * q)) : 0u;
                 hi_w = 0u;
             } else {
-                lo_w = (jj < nb && e < 4) ? (best_o << (8 * e)) : 0u;
-                hi_w = (jj < nb && e >= 4) ? (best_o << (8 * (e - 4))) : 0u;
+                lo_w = (jj < g.nb && q < 4) ? (best_o << (8 * q)) : 0u;
+                hi_w = (jj < g.nb && q >= 4) ? (best_o << (8 * (q - 4))) : 0u;
             }
 #pragma unroll
             for (int d = 1; d < kChunk; d <<= 1) {
                 lo_w |= __shfl_xor_sync(0xFFFFFFFFu, lo_w, d);
                 hi_w |= __shfl_xor_sync(0xFFFFFFFFu, hi_w, d);
             }
-            if (e == 0 && jj < nb) {
-                const int64_t rec = static_cast<int64_t>(j / kChunk) * kSlots + slot;
-                if (grp.nib) {
-                    t.offs[grp.off_off + rec] = lo_w;
-                } else {
-                    reinterpret_cast<uint2 *>(t.offs + grp.off_off)[rec] = make_uint2(lo_w, hi_w);
-                }
+            if (q == 0 && jj < g.nb) {
+                const int64_t rec = int64_t(j / kChunk) * kSlots + slot;
+                if (grp.nib) t.offs[grp.off_off + rec] = lo_w;
+                else reinterpret_cast<uint2 *>(t.offs + grp.off_off)[rec] = make_uint2(lo_w, hi_w);
             }
         }
+        __syncthreads();   // this stage is free for the copy issued next iteration
     }
-    if (__syncthreads_or(nan) && threadIdx.x == 0) atomicExch(err_flag, 1);
+    if (!ok) {
+        // a copy did not land in time: record it and let the copies still in flight settle
+        if (tid == 0) atomicOr(status, kStatusTimeout);
+        for (int k = 1; k < kStages; ++k) {
+            const int s = (it + k) % kStages;
+            mbar_wait(&bar[s], (phases >> s) & 1u);
+        }
+    }
+    if (__syncthreads_or(nan) && tid == 0) atomicOr(status, kStatusNaN);
 }
 
 }  // namespace
 
-cudaError_t launch_encode(const EncodeTarget &t, const void *W, int64_t ldw, int32_t *err_flag,
+cudaError_t launch_encode(const EncodeTarget &t, const void *W, int64_t ldw, int32_t *status,
                           cudaStream_t stream) {
-    dim3 grid(static_cast<unsigned>(t.rows));
+    const int per_sm = t.bf16 ? 3 : 2;   // resident CTAs per SM at this kernel's shared memory
+    const unsigned grid = static_cast<unsigned>(std::min<int64_t>(t.ntiles, per_sm * int64_t(sm_count())));
+    if (grid == 0) return cudaSuccess;
     if (t.bf16) {
-        encode_kernel<true><<<grid, kEncThreads, 0, stream>>>(t, W, ldw, err_flag);
-    } else {
-        encode_kernel<false><<<grid, kEncThreads, 0, stream>>>(t, W, ldw, err_flag);
+        static const cudaError_t a = allow_smem(encode_kernel<true>, encode_smem<true>());
+        if (a != cudaSuccess) return a;
+        return launch_ex(encode_kernel<true>, dim3(grid), dim3(kEncThreads), encode_smem<true>(), stream,
+                         1, true, t, W, ldw, status);
     }
-    return cudaGetLastError();
+    static const cudaError_t a = allow_smem(encode_kernel<false>, encode_smem<false>());
+    if (a != cudaSuccess) return a;
+    return launch_ex(encode_kernel<false>, dim3(grid), dim3(kEncThreads), encode_smem<false>(), stream,
+                     1, true, t, W, ldw, status);
 }
 
 }  // namespace darb

@@ -15,6 +15,8 @@
 // GRU keeps the x-part and h-part of each gate sum apart (a and bh), since the
 // reset gate multiplies only the h-part of the candidate gate.
 #include "kernels_common.cuh"
+#include "launch.cuh"
+#include "tma.cuh"
 
 namespace darb {
 namespace {
@@ -34,6 +36,8 @@ __global__ void __launch_bounds__(kWarps * 32)
 rnn_step_rowlane(Format f, XStacked xs, int64_t B, int H, RnnScratch sc, CellArgs ca) {
     constexpr int kParts = GRU ? 2 : 1;
     __shared__ float red[kWarps][kSlots][BT * kParts];
+    pdl_launch_dependents();
+    pdl_wait_previous();
     const int gi = blockIdx.x;
     const Group g = f.groups[gi];
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -123,20 +127,19 @@ cudaError_t launch_step(const Format &f, int64_t I, int64_t H, int64_t B, const 
     const dim3 grid(static_cast<unsigned>(f.ngroups), static_cast<unsigned>((B + bt - 1) / bt));
     const dim3 block(kWarps * 32);
     const int h = static_cast<int>(H);
-#define DARB_STEP(BF, BTV) rnn_step_rowlane<BF, BTV, GRU><<<grid, block, 0, stream>>>(f, xs, B, h, sc, ca)
+#define DARB_STEP(BF, BTV) \
+    launch_ex(rnn_step_rowlane<BF, BTV, GRU>, grid, block, 0, stream, 1, true, f, xs, B, h, sc, ca)
     if (f.bf16) {
-        if (bt == 1) DARB_STEP(true, 1);
-        else if (bt == 2) DARB_STEP(true, 2);
-        else if (bt == 4) DARB_STEP(true, 4);
-        else DARB_STEP(true, 8);
-    } else {
-        if (bt == 1) DARB_STEP(false, 1);
-        else if (bt == 2) DARB_STEP(false, 2);
-        else if (bt == 4) DARB_STEP(false, 4);
-        else DARB_STEP(false, 8);
+        if (bt == 1) return DARB_STEP(true, 1);
+        if (bt == 2) return DARB_STEP(true, 2);
+        if (bt == 4) return DARB_STEP(true, 4);
+        return DARB_STEP(true, 8);
     }
+    if (bt == 1) return DARB_STEP(false, 1);
+    if (bt == 2) return DARB_STEP(false, 2);
+    if (bt == 4) return DARB_STEP(false, 4);
+    return DARB_STEP(false, 8);
 #undef DARB_STEP
-    return cudaGetLastError();
 }
 
 }  // namespace

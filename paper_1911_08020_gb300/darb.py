@@ -53,7 +53,7 @@ def lib():
                 "darb_assign_block_sizes": [P, I64, I64, I32, I32, P],
                 "darb_encode": [P, ctypes.c_int, I64, I64, I64, P, P, S],
                 "darb_reencode": [P, P, I64, S],
-                "darb_encode_status": [P, S],
+                "darb_sync_status": [P, S],
                 "darb_spmm": [P, P, I64, I64, P, I64, S],
                 "darb_lstm_step": [P, I64, I64, I64, P, P, P, P, P, P, S],
                 "darb_gru_step": [P, I64, I64, I64, P, P, P, P, P, S],
@@ -157,8 +157,9 @@ def darb_reencode(h: Handle, W, stream=None):
     _check(lib().darb_reencode(h.ptr, _ptr(W), W.stride(0), _stream(stream)), "darb_reencode")
 
 
-def darb_encode_status(h: Handle, stream=None):
-    _check(lib().darb_encode_status(h.ptr, _stream(stream)), "darb_encode_status")
+def darb_sync_status(h: Handle, stream=None):
+    """Synchronise and raise if the handle's kernels recorded a NaN or a timeout."""
+    _check(lib().darb_sync_status(h.ptr, _stream(stream)), "darb_sync_status")
 
 
 def darb_spmm(h: Handle, X, Y=None, stream=None):

@@ -128,15 +128,15 @@ def test_reencode_and_status():
     h = darb.darb_encode(t(w1), m)
     try:
         darb.darb_reencode(h, t(w2))
-        darb.darb_encode_status(h)
+        darb.darb_sync_status(h)
         assert_encoding_equal(h, oracle.encode(w2, m))
         w3 = w2.copy()
         w3[5, 5] = np.nan
         darb.darb_reencode(h, t(w3))
         with pytest.raises(darb.DarbError) as e:
-            darb.darb_encode_status(h)
+            darb.darb_sync_status(h)
         assert e.value.status == darb.ERR_NONFINITE
-        darb.darb_encode_status(h)   # flag cleared
+        darb.darb_sync_status(h)   # flag cleared
     finally:
         darb.darb_destroy(h)
 
