@@ -27,12 +27,15 @@ struct darb_handle_s {
     std::vector<Group> groups;
     std::vector<int32_t> rowmap, rowloc, row_m;
     std::vector<int2> enc_tiles;   // (row, first block) of every encoder tile
+    std::vector<int2> sets;        // row sets of up to 1, 2, 4, 8 groups, concatenated
+    int32_t nsets[4] = {0, 0, 0, 0};
     int64_t val_elems = 0, off_words = 0;
     // device memory: one allocation holding the layout, values and offsets
     void *dmem = nullptr;
     size_t dbytes = 0;
     Group *d_groups = nullptr;
     int2 *d_tiles = nullptr;
+    int2 *d_sets = nullptr;
     int32_t *d_rowmap = nullptr, *d_rowloc = nullptr, *d_row_m = nullptr, *d_status = nullptr;
     void *d_vals = nullptr;
     uint32_t *d_offs = nullptr;
@@ -136,6 +139,22 @@ void build_layout(darb_handle_s *h, const int32_t *m) {
     }
     h->val_elems = val;
     h->off_words = off;
+    // row sets: consecutive groups of one bin, at most 2^i per set
+    h->sets.clear();
+    for (int i = 0; i < 4; ++i) {
+        const int cap = 1 << i;
+        h->nsets[i] = 0;
+        size_t gbeg = 0;
+        while (gbeg < h->groups.size()) {
+            size_t gend = gbeg;
+            while (gend < h->groups.size() && h->groups[gend].m == h->groups[gbeg].m) ++gend;
+            for (size_t s = gbeg; s < gend; s += cap) {
+                h->sets.push_back(make_int2(static_cast<int>(s), static_cast<int>(std::min<size_t>(cap, gend - s))));
+                ++h->nsets[i];
+            }
+            gbeg = gend;
+        }
+    }
     h->enc_tiles.clear();
     for (int64_t r = 0; r < rows; ++r) {
         const int tb = darb::enc_tile_blocks(m[r]);
@@ -150,6 +169,7 @@ darb_status_t alloc_device(darb_handle_s *h) {
     size_t o = 0;
     const size_t o_groups = o; o = align_up(o + h->groups.size() * sizeof(Group), 256);
     const size_t o_tiles = o;  o = align_up(o + h->enc_tiles.size() * sizeof(int2), 256);
+    const size_t o_sets = o;   o = align_up(o + h->sets.size() * sizeof(int2), 256);
     const size_t o_rowmap = o; o = align_up(o + h->rowmap.size() * 4, 256);
     const size_t o_rowloc = o; o = align_up(o + h->rowloc.size() * 4, 256);
     const size_t o_rowm = o;   o = align_up(o + h->row_m.size() * 4, 256);
@@ -164,6 +184,7 @@ darb_status_t alloc_device(darb_handle_s *h) {
     h->dbytes = o;
     h->d_groups = reinterpret_cast<Group *>(b + o_groups);
     h->d_tiles = reinterpret_cast<int2 *>(b + o_tiles);
+    h->d_sets = reinterpret_cast<int2 *>(b + o_sets);
     h->d_rowmap = reinterpret_cast<int32_t *>(b + o_rowmap);
     h->d_rowloc = reinterpret_cast<int32_t *>(b + o_rowloc);
     h->d_row_m = reinterpret_cast<int32_t *>(b + o_rowm);
@@ -180,6 +201,9 @@ darb_status_t upload_layout(darb_handle_s *h, cudaStream_t stream) {
                             cudaMemcpyHostToDevice, stream);
     if (e == cudaSuccess)
         e = cudaMemcpyAsync(h->d_tiles, h->enc_tiles.data(), h->enc_tiles.size() * sizeof(int2),
+                            cudaMemcpyHostToDevice, stream);
+    if (e == cudaSuccess)
+        e = cudaMemcpyAsync(h->d_sets, h->sets.data(), h->sets.size() * sizeof(int2),
                             cudaMemcpyHostToDevice, stream);
     if (e == cudaSuccess)
         e = cudaMemcpyAsync(h->d_rowmap, h->rowmap.data(), h->rowmap.size() * 4,
@@ -216,6 +240,10 @@ Format format_of(const darb_handle_s *h) {
     f.vals = h->d_vals;
     f.offs = h->d_offs;
     f.status = h->d_status;
+    for (int i = 0, o = 0; i < 4; o += h->nsets[i], ++i) {
+        f.sets[i] = h->d_sets + o;
+        f.nsets[i] = h->nsets[i];
+    }
     f.ngroups = static_cast<int32_t>(h->groups.size());
     f.bf16 = h->wtype == DARB_BF16 ? 1 : 0;
     f.rows = h->rows;

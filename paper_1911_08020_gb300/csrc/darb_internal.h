@@ -50,6 +50,10 @@ struct Format {
     const void *vals;        // fp32 or bf16 bit patterns
     const uint32_t *offs;
     int32_t *status;         // sticky device status bits (NaN seen, wait timed out)
+    // row sets: runs of up to 1, 2, 4, 8 consecutive groups of one bin, as
+    // (first group, group count); sets[i] holds the sets of up to 2^i groups
+    const int2 *sets[4];
+    int32_t nsets[4];
     int32_t ngroups;
     int32_t bf16;            // value dtype: 0 fp32, 1 bf16
     int64_t rows, cols;
@@ -76,6 +80,10 @@ struct RnnScratch {
 
 cudaError_t launch_encode(const EncodeTarget &t, const void *W, int64_t ldw, int32_t *status,
                           cudaStream_t stream);
+
+// Batch > 4 path (spmm_batch.cu).
+cudaError_t launch_spmm_batch(const Format &f, const float *X, int64_t ldx, int64_t batch, float *Y,
+                              int64_t ldy, bool early, cudaStream_t stream);
 
 // `early`: the handle's data is known to be complete, so a kernel may start
 // reading it before the previous kernel on the stream has finished (PDL).
