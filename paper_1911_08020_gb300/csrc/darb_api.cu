@@ -246,6 +246,7 @@ Format format_of(const darb_handle_s *h) {
     }
     f.ngroups = static_cast<int32_t>(h->groups.size());
     f.bf16 = h->wtype == DARB_BF16 ? 1 : 0;
+    f.m_max = h->groups.empty() ? 1 : h->groups.back().m;
     f.rows = h->rows;
     f.cols = h->cols;
     return f;

@@ -34,31 +34,47 @@ namespace cg = cooperative_groups;
 namespace darb {
 namespace {
 
-constexpr int kXcapB = 8192;      // activation floats per round (before box slack)
-constexpr int kBoxRows = 64;      // rows per 2-D tensor copy
-constexpr int kRecCap = 32;       // (group, chunk) records staged per round
-constexpr int kMaxSetGroups = 8;
+constexpr int kXcapB = 8192;      // activation floats per round
+constexpr int kXslack = 2048;     // room for the last tensor box of a round to run past it
+constexpr int kXstage = kXcapB + kXslack;
+constexpr int kRecCap = 16;       // (group, chunk) records staged per round
+constexpr int kStages = 2;        // rounds in flight per CTA
 
-template <bool BF16, int LPR>
+// Lanes per row LPR, columns per lane CPL: the batch tile is LPR*CPL columns.
+// Wide tiles keep fewer rows per set so that the accumulators fit in registers.
+template <int LPR, int CPL>
+__host__ __device__ constexpr int max_set_groups() { return CPL == 8 ? 4 : 8; }
+
+template <int LPR, int CPL>
+__host__ __device__ constexpr int box_rows() { return kXslack / (LPR * CPL); }
+
+template <bool BF16>
+__host__ __device__ constexpr size_t stage_val_bytes() { return size_t(kRecCap) * kSlots * kChunk * (BF16 ? 2 : 4); }
+
+constexpr size_t kStageOffBytes = size_t(kRecCap) * kSlots * 2 * 4;
+
+template <bool BF16>
 __host__ __device__ constexpr size_t batch_smem() {
-    return 128 + size_t(kXcapB + kBoxRows * 4 * LPR) * 4 + size_t(kRecCap) * kSlots * kChunk * (BF16 ? 2 : 4) +
-           size_t(kRecCap) * kSlots * 2 * 4;
+    return 128 + kStages * (size_t(kXstage) * 4 + stage_val_bytes<BF16>() + kStageOffBytes);
 }
 
-template <bool BF16, int LPR>
+template <bool BF16, int LPR, int CPL>
 __global__ void __launch_bounds__(kWarps * 32)
 spmm_batch(Format f, const int2 *__restrict__ sets, const float *__restrict__ X, int64_t ldx, int64_t batch,
            float *__restrict__ Y, int64_t ldy, const __grid_constant__ CUtensorMap xmap, int use_tma,
            int early) {
-    constexpr int kBt = 4 * LPR;          // batch tile
+    constexpr int kBt = LPR * CPL;        // batch tile
+    constexpr int kQ = CPL / 4;           // float4 per lane
     constexpr int kRpw = 32 / LPR;        // rows per warp at a time
-    constexpr int kRptMax = kMaxSetGroups * kSlots / (kWarps * kRpw);
+    constexpr int kRptMax = max_set_groups<LPR, CPL>() * kSlots / (kWarps * kRpw);
+    constexpr int kBoxRows = box_rows<LPR, CPL>();
     constexpr int kEsz = BF16 ? 2 : 4;
     extern __shared__ __align__(128) unsigned char sm[];
+    // layout: barriers | X stage 0 | X stage 1 | values x2 | offsets x2
     uint64_t *bar = reinterpret_cast<uint64_t *>(sm);
-    float *s_x = reinterpret_cast<float *>(sm + 128);   // activation tile, later partial sums
-    unsigned char *s_vals = sm + 128 + size_t(kXcapB + kBoxRows * kBt) * 4;
-    uint32_t *s_offs = reinterpret_cast<uint32_t *>(s_vals + size_t(kRecCap) * kSlots * kChunk * kEsz);
+    float *s_x0 = reinterpret_cast<float *>(sm + 128);
+    unsigned char *s_v0 = sm + 128 + size_t(kStages) * kXstage * 4;
+    unsigned char *s_o0 = s_v0 + kStages * stage_val_bytes<BF16>();
 
     pdl_launch_dependents();
     cg::cluster_group cluster = cg::this_cluster();
@@ -80,73 +96,92 @@ spmm_batch(Format f, const int2 *__restrict__ sets, const float *__restrict__ X,
     const int rounds = (J1 - J0 + rb - 1) / rb;
 
     if (tid == 0) {
-        mbar_init(bar, 1);
+        for (int st = 0; st < kStages; ++st) mbar_init(&bar[st], 1);
         fence_mbar_init();
     }
     __syncthreads();
 
-    auto round_geo = [&](int r, int &jr0, int &jr1, int &cr0, int &nchr) {
-        jr0 = J0 + r * rb;
-        jr1 = min(J1, jr0 + rb);
-        cr0 = jr0 / kChunk;
-        nchr = (jr1 + kChunk - 1) / kChunk - cr0;
+    struct Round { int jr0, jr1, cr0, nchr, kx0, kr; };
+    auto round_geo = [&](int r) {
+        Round g;
+        g.jr0 = J0 + r * rb;
+        g.jr1 = min(J1, g.jr0 + rb);
+        g.cr0 = g.jr0 / kChunk;
+        g.nchr = (g.jr1 + kChunk - 1) / kChunk - g.cr0;
+        g.kx0 = g.jr0 * m;
+        const int64_t kxe = int64_t(g.jr1) * m;
+        g.kr = static_cast<int>((kxe < f.cols ? kxe : f.cols) - g.kx0);
+        return g;
     };
-    // copies of the handle's values and offsets for round r (thread 0)
-    auto issue_handle = [&](int r, bool arrive, uint32_t extra) {
-        int jr0, jr1, cr0, nchr;
-        round_geo(r, jr0, jr1, cr0, nchr);
-        const uint32_t bv = uint32_t(nchr) * kSlots * kChunk * kEsz;
-        const uint32_t bo = uint32_t(nchr) * kSlots * rw * 4;
-        if (arrive) mbar_arrive_expect_tx(bar, uint32_t(ng) * (bv + bo) + extra);
-        else mbar_expect_tx(bar, uint32_t(ng) * (bv + bo));
-        for (int gi = 0; gi < ng; ++gi) {
-            const Group g = f.groups[set.x + gi];
-            bulk_g2s(s_vals + size_t(gi) * bv,
-                     static_cast<const unsigned char *>(f.vals) + (size_t(g.val_off) + size_t(cr0) * kSlots * kChunk) * kEsz,
-                     bv, bar);
-            bulk_g2s(reinterpret_cast<unsigned char *>(s_offs) + size_t(gi) * bo,
-                     f.offs + g.off_off + size_t(cr0) * kSlots * rw, bo, bar);
-        }
-    };
-    if (early && rounds > 0 && tid == 0) issue_handle(0, false, 0);
-    pdl_wait_previous();
-
-    float4 acc[kRptMax];
-#pragma unroll
-    for (int p = 0; p < kRptMax; ++p) acc[p] = make_float4(0.f, 0.f, 0.f, 0.f);
-    const int rpt = (ng * kSlots + kWarps * kRpw - 1) / (kWarps * kRpw);
-    bool ok = true;
-    int r_fail = 0;
-    for (int r = 0; r < rounds && ok; ++r) {
-        r_fail = r;
-        int jr0, jr1, cr0, nchr;
-        round_geo(r, jr0, jr1, cr0, nchr);
-        const int kx0 = jr0 * m;
-        const int64_t kxe = int64_t(jr1) * m;
-        const int kr = static_cast<int>((kxe < f.cols ? kxe : f.cols) - kx0);
-        const int nbox = (kr + kBoxRows - 1) / kBoxRows;
-        if (tid == 0) {
-            if (r > 0) fence_proxy_async_smem();   // last round's generic reads come first
-            const uint32_t xbytes = use_tma ? uint32_t(nbox) * kBoxRows * kBt * 4 : 0u;
-            if (early && r == 0) {
-                mbar_arrive_expect_tx(bar, xbytes);
-            } else {
-                issue_handle(r, true, xbytes);
+    // Thread 0 starts round r's copies into stage st.  The handle part (kept
+    // values and offsets, per group one contiguous run each) may go before the
+    // PDL wait; the activation part only after it.  Exactly one arrival per
+    // round closes the stage's phase together with the transferred bytes.
+    auto issue = [&](int r, int st, bool handle, bool xpart) {
+        const Round g = round_geo(r);
+        const uint32_t bv = uint32_t(g.nchr) * kSlots * kChunk * kEsz;
+        const uint32_t bo = uint32_t(g.nchr) * kSlots * rw * 4;
+        const int nbox = (g.kr + kBoxRows - 1) / kBoxRows;
+        const uint32_t hbytes = handle ? uint32_t(ng) * (bv + bo) : 0u;
+        const uint32_t xbytes = (xpart && use_tma) ? uint32_t(nbox) * kBoxRows * kBt * 4 : 0u;
+        if (xpart) mbar_arrive_expect_tx(&bar[st], hbytes + xbytes);
+        else mbar_expect_tx(&bar[st], hbytes);
+        if (handle)
+            for (int gi = 0; gi < ng; ++gi) {
+                const Group gg = f.groups[set.x + gi];
+                bulk_g2s(s_v0 + st * stage_val_bytes<BF16>() + size_t(gi) * bv,
+                         static_cast<const unsigned char *>(f.vals) +
+                             (size_t(gg.val_off) + size_t(g.cr0) * kSlots * kChunk) * kEsz,
+                         bv, &bar[st]);
+                bulk_g2s(s_o0 + st * kStageOffBytes + size_t(gi) * bo,
+                         f.offs + gg.off_off + size_t(g.cr0) * kSlots * rw, bo, &bar[st]);
             }
-            if (use_tma)
-                for (int i = 0; i < nbox; ++i)
-                    tensor2d_g2s(s_x + size_t(i) * kBoxRows * kBt, &xmap, int(b0), kx0 + i * kBoxRows, bar);
-        }
+        if (xpart && use_tma)
+            for (int i = 0; i < nbox; ++i)
+                tensor2d_g2s(s_x0 + size_t(st) * kXstage + size_t(i) * kBoxRows * kBt, &xmap, int(b0),
+                             g.kx0 + i * kBoxRows, &bar[st]);
+    };
+    const int pre = min(rounds, kStages);
+    if (early && tid == 0)
+        for (int r = 0; r < pre; ++r) issue(r, r, true, false);
+    pdl_wait_previous();
+    if (tid == 0)
+        for (int r = 0; r < pre; ++r) issue(r, r, !early, true);
+
+    float4 acc[kRptMax][kQ];
+#pragma unroll
+    for (int p = 0; p < kRptMax; ++p)
+#pragma unroll
+        for (int u = 0; u < kQ; ++u) acc[p][u] = make_float4(0.f, 0.f, 0.f, 0.f);
+    const int rpt = (ng * kSlots + kWarps * kRpw - 1) / (kWarps * kRpw);
+    // which of this thread's row slots hold a matrix row
+    uint32_t valid_mask = 0u;
+#pragma unroll
+    for (int p = 0; p < kRptMax; ++p) {
+        const int s = warp * kRpw + rr + p * kWarps * kRpw;
+        const int gi = s / kSlots;
+        if (p < rpt && gi < ng && (s % kSlots) < f.groups[set.x + gi].nrows) valid_mask |= 1u << p;
+    }
+    bool ok = true;
+    int r_last = 0;
+    // round r uses stage r % kStages for the (r / kStages)-th time: that is its phase parity
+    for (int r = 0; r < rounds && ok; ++r) {
+        r_last = r;
+        const int st = r % kStages;
+        const Round g = round_geo(r);
+        float *s_x = s_x0 + size_t(st) * kXstage;
+        const unsigned char *s_vals = s_v0 + st * stage_val_bytes<BF16>();
+        const uint32_t *s_offs = reinterpret_cast<const uint32_t *>(s_o0 + st * kStageOffBytes);
         if (!use_tma) {
             // X not addressable by a tensor map: 8 independent loads in flight per thread
-            const int nx = kr * kBt;
+            const int nx = g.kr * kBt;
             for (int base = 0; base < nx; base += 8 * kWarps * 32) {
                 float tmp[8];
 #pragma unroll
                 for (int u = 0; u < 8; ++u) {
                     const int idx = base + u * kWarps * 32 + tid;
                     const int kk = idx / kBt, t = idx % kBt;
-                    tmp[u] = (idx < nx && b0 + t < batch) ? __ldg(X + int64_t(kx0 + kk) * ldx + b0 + t) : 0.0f;
+                    tmp[u] = (idx < nx && b0 + t < batch) ? __ldg(X + int64_t(g.kx0 + kk) * ldx + b0 + t) : 0.0f;
                 }
 #pragma unroll
                 for (int u = 0; u < 8; ++u) {
@@ -154,20 +189,21 @@ spmm_batch(Format f, const int2 *__restrict__ sets, const float *__restrict__ X,
                     if (idx < nx) s_x[idx] = tmp[u];
                 }
             }
+            __syncthreads();
         }
-        __syncthreads();
-        ok = __syncthreads_and(mbar_wait(bar, r & 1));
+        ok = __syncthreads_and(mbar_wait(&bar[st], (r / kStages) & 1));
         if (ok) {
             const float4 *sx4 = reinterpret_cast<const float4 *>(s_x);
-            for (int lc = 0; lc < nchr; ++lc) {
-                const int jc = (cr0 + lc) * kChunk;
+            for (int lc = 0; lc < g.nchr; ++lc) {
+                const int jc = (g.cr0 + lc) * kChunk;
+                // blocks of this chunk inside the round (all 8 except at the round's ends)
+                const int e_lo = max(0, g.jr0 - jc), e_hi = min(kChunk, g.jr1 - jc);
+                const bool whole = e_lo == 0 && e_hi == kChunk;
 #pragma unroll
                 for (int p = 0; p < kRptMax; ++p) {
-                    const int s = warp * kRpw + rr + p * kWarps * kRpw;
-                    const int gi = s / kSlots, slot = s % kSlots;
-                    const bool valid = p < rpt && gi < ng && slot < f.groups[set.x + min(gi, ng - 1)].nrows;
-                    if (valid) {
-                        const int rec = (gi * nchr + lc) * kSlots + slot;
+                    if (valid_mask & (1u << p)) {
+                        const int s = warp * kRpw + rr + p * kWarps * kRpw;
+                        const int rec = ((s / kSlots) * g.nchr + lc) * kSlots + (s % kSlots);
                         float v[kChunk];
                         if constexpr (BF16) {
                             const uint4 w4 = *reinterpret_cast<const uint4 *>(s_vals + size_t(rec) * 16);
@@ -186,38 +222,53 @@ spmm_batch(Format f, const int2 *__restrict__ sets, const float *__restrict__ X,
                         uint2 ow;
                         if (rw == 1) ow = make_uint2(s_offs[rec], 0u);
                         else ow = reinterpret_cast<const uint2 *>(s_offs)[rec];
+                        // lane qd owns float4 columns u*LPR + qd: for each u a
+                        // quarter-warp reads 128 contiguous bytes (no conflicts)
+                        const float4 *xb = sx4 + (jc * m - g.kx0) * (kBt / 4) + qd;
 #pragma unroll
                         for (int e = 0; e < kChunk; ++e) {
-                            const int j = jc + e;
-                            if (j >= jr0 && j < jr1) {
+                            if (whole || (e >= e_lo && e < e_hi)) {
                                 const int off = rw == 1 ? int((ow.x >> (4 * e)) & 15u)
                                                         : int(((e < 4 ? ow.x : ow.y) >> (8 * (e & 3))) & 255u);
-                                const float4 xv = sx4[(j * m + off - kx0) * LPR + qd];
-                                acc[p].x = fmaf(v[e], xv.x, acc[p].x);
-                                acc[p].y = fmaf(v[e], xv.y, acc[p].y);
-                                acc[p].z = fmaf(v[e], xv.z, acc[p].z);
-                                acc[p].w = fmaf(v[e], xv.w, acc[p].w);
+                                const float4 *xr = xb + (e * m + off) * (kBt / 4);
+#pragma unroll
+                                for (int u = 0; u < kQ; ++u) {
+                                    const float4 xv = xr[u * LPR];
+                                    acc[p][u].x = fmaf(v[e], xv.x, acc[p][u].x);
+                                    acc[p][u].y = fmaf(v[e], xv.y, acc[p][u].y);
+                                    acc[p][u].z = fmaf(v[e], xv.z, acc[p][u].z);
+                                    acc[p][u].w = fmaf(v[e], xv.w, acc[p][u].w);
+                                }
                             }
                         }
                     }
                 }
             }
         }
-        __syncthreads();
+        __syncthreads();   // stage st is free again
+        if (ok && r + kStages < rounds && tid == 0) {
+            fence_proxy_async_smem();
+            issue(r + kStages, st, true, true);
+        }
     }
     if (!ok) {
-        // a copy did not land in time: record it, let in-flight copies settle,
-        // and finish without trusting the sums
+        // a copy did not land in time: record it, let the copies still in
+        // flight settle, and finish without trusting the sums
         if (tid == 0) atomicOr(f.status, kStatusTimeout);
-        mbar_wait(bar, r_fail & 1);
+        for (int r = r_last; r < min(rounds, r_last + kStages); ++r)
+            mbar_wait(&bar[r % kStages], (r / kStages) & 1);
         __syncthreads();
     }
-    // partial sums of every row slot of the set, slot-major: part[s][0..kBt)
-    float4 *part4 = reinterpret_cast<float4 *>(s_x);
+    // partial sums of every row slot of the set, slot-major: part[s][0..kBt),
+    // over both X stages (contiguous)
+    float *part = s_x0;
+    float4 *part4 = reinterpret_cast<float4 *>(part);
 #pragma unroll
     for (int p = 0; p < kRptMax; ++p) {
         const int s = warp * kRpw + rr + p * kWarps * kRpw;
-        if (p < rpt && s < ng * kSlots) part4[s * LPR + qd] = acc[p];
+        if (p < rpt && s < ng * kSlots)
+#pragma unroll
+            for (int u = 0; u < kQ; ++u) part4[s * (kBt / 4) + u * LPR + qd] = acc[p][u];
     }
     __syncthreads();
     if (ksc > 1) cluster.sync();
@@ -230,7 +281,7 @@ spmm_batch(Format f, const int2 *__restrict__ sets, const float *__restrict__ X,
         const int gi = s / kSlots, slot = s % kSlots;
         if (b0 + t >= batch || slot >= f.groups[set.x + gi].nrows) continue;
         float sum = 0.0f;   // ranks in a fixed order: deterministic
-        for (int r = 0; r < ksc; ++r) sum += cluster.map_shared_rank(s_x, r)[s * kBt + t];
+        for (int r = 0; r < ksc; ++r) sum += cluster.map_shared_rank(part, r)[s * kBt + t];
         const int row = f.rowmap[(set.x + gi) * kSlots + slot];
         Y[int64_t(row) * ldy + b0 + t] = sum;
     }
@@ -252,49 +303,61 @@ PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
 }
 
 // Tensor map over X (cols rows of `batch` floats, row pitch ldx) with a
-// kBoxRows x bt box; false if X cannot be described (alignment).
-bool make_xmap(CUtensorMap *map, const float *X, int64_t ldx, int64_t batch, int64_t cols, int bt) {
+// boxr x bt box; false if X cannot be described (alignment).
+bool make_xmap(CUtensorMap *map, const float *X, int64_t ldx, int64_t batch, int64_t cols, int bt,
+               int boxr) {
     if (reinterpret_cast<uintptr_t>(X) % 16 != 0 || (ldx * 4) % 16 != 0) return false;
     PFN_cuTensorMapEncodeTiled_v12000 enc = tensor_map_encoder();
     if (enc == nullptr) return false;
     const cuuint64_t dims[2] = {cuuint64_t(batch), cuuint64_t(cols)};
     const cuuint64_t strides[1] = {cuuint64_t(ldx) * 4};
-    const cuuint32_t box[2] = {cuuint32_t(bt), cuuint32_t(kBoxRows)};
+    const cuuint32_t box[2] = {cuuint32_t(bt), cuuint32_t(boxr)};
     const cuuint32_t estr[2] = {1, 1};
     return enc(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, const_cast<float *>(X), dims, strides, box, estr,
                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-template <bool BF16, int LPR>
+template <bool BF16, int LPR, int CPL>
 cudaError_t launch_batch(const Format &f, const float *X, int64_t ldx, int64_t batch, float *Y,
                          int64_t ldy, bool early, cudaStream_t stream) {
-    constexpr int kBt = 4 * LPR;
-    constexpr size_t smem = batch_smem<BF16, LPR>();
-    static const cudaError_t attr = allow_smem(spmm_batch<BF16, LPR>, smem);
+    constexpr int kBt = LPR * CPL;
+    constexpr size_t smem = batch_smem<BF16>();
+    static const cudaError_t attr = allow_smem(spmm_batch<BF16, LPR, CPL>, smem);
     if (attr != cudaSuccess) return attr;
     CUtensorMap map;
     std::memset(&map, 0, sizeof map);
-    const int use_tma = make_xmap(&map, X, ldx, batch, f.cols, kBt) ? 1 : 0;
-    const int level = 3;   // sets of up to 8 groups
+    const int use_tma = make_xmap(&map, X, ldx, batch, f.cols, kBt, box_rows<LPR, CPL>()) ? 1 : 0;
     const int64_t tiles = (batch + kBt - 1) / kBt;
-    // cluster split so that the grid fills the GPU about twice over
+    const int64_t target = 3 * int64_t(sm_count());   // CTAs wanted
+    // largest row sets (most reuse of each staged activation row) that still
+    // give enough CTAs with a cluster split of at most 8
+    int level = 0;
+    for (int l = 3; l >= 0; --l) {
+        if ((1 << l) > max_set_groups<LPR, CPL>()) continue;
+        level = l;
+        if (int64_t(f.nsets[l]) * tiles * 8 >= target) break;
+    }
     unsigned ksc = 1;
-    while (ksc < 8 && int64_t(f.nsets[level]) * tiles * ksc * 2 <= 3 * int64_t(sm_count())) ksc *= 2;
+    while (ksc < 8 && int64_t(f.nsets[level]) * tiles * ksc < target) ksc *= 2;
     const dim3 grid(static_cast<unsigned>(f.nsets[level]) * ksc, static_cast<unsigned>(tiles));
-    return launch_ex(spmm_batch<BF16, LPR>, grid, dim3(kWarps * 32), smem, stream, ksc, true, f, f.sets[level], X,
-                     ldx, batch, Y, ldy, map, use_tma, early ? 1 : 0);
+    return launch_ex(spmm_batch<BF16, LPR, CPL>, grid, dim3(kWarps * 32), smem, stream, ksc, true, f,
+                     f.sets[level], X, ldx, batch, Y, ldy, map, use_tma, early ? 1 : 0);
 }
 
 }  // namespace
 
 cudaError_t launch_spmm_batch(const Format &f, const float *X, int64_t ldx, int64_t batch, float *Y,
                               int64_t ldy, bool early, cudaStream_t stream) {
-    if (batch <= 16)
-        return f.bf16 ? launch_batch<true, 4>(f, X, ldx, batch, Y, ldy, early, stream)
-                      : launch_batch<false, 4>(f, X, ldx, batch, Y, ldy, early, stream);
-    return f.bf16 ? launch_batch<true, 8>(f, X, ldx, batch, Y, ldy, early, stream)
-                  : launch_batch<false, 8>(f, X, ldx, batch, Y, ldy, early, stream);
+    // one block's activation rows (m_max of them) must fit a stage's tile
+    if (batch <= 16 || int64_t(f.m_max) * 32 > kXcapB)
+        return f.bf16 ? launch_batch<true, 4, 4>(f, X, ldx, batch, Y, ldy, early, stream)
+                      : launch_batch<false, 4, 4>(f, X, ldx, batch, Y, ldy, early, stream);
+    if (batch <= 32 || int64_t(f.m_max) * 64 > kXcapB)
+        return f.bf16 ? launch_batch<true, 8, 4>(f, X, ldx, batch, Y, ldy, early, stream)
+                      : launch_batch<false, 8, 4>(f, X, ldx, batch, Y, ldy, early, stream);
+    return f.bf16 ? launch_batch<true, 8, 8>(f, X, ldx, batch, Y, ldy, early, stream)
+                  : launch_batch<false, 8, 8>(f, X, ldx, batch, Y, ldy, early, stream);
 }
 
 }  // namespace darb
