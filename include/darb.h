@@ -166,6 +166,31 @@ DARB_API darb_status_t darb_gru_step(darb_handle_t h, int64_t I, int64_t H, int6
                             const float *h_prev, const float *b_ih, const float *b_hh,
                             float *h_out, cudaStream_t stream);
 
+/*
+ * darb_lstm_step without any allocation: the same step, same arguments and
+ * same results, with its scratch (gate sums and arrival counters) in one
+ * fixed array of 4 MiB inside this library instead of memory owned by the
+ * handle.  It is for callers that cannot let a library call cudaMalloc at step
+ * time -- a serving loop with a fixed memory budget, code that must not
+ * synchronise the device mid-stream, or allocations that must all go through
+ * the caller's own pool.  The paper has no counterpart; it is a property of
+ * this library's interface only.
+ *   - Limit: 4H*B floats (rounded up to 256 bytes) plus H*ceil(B/t) counters
+ *     (t = 1, 2, 4 or 8 by batch) must fit in 4 MiB; larger calls return
+ *     DARB_ERR_UNSUPPORTED and do nothing.
+ *   - Every GPU that loads the library holds the 4 MiB until the process exits.
+ *   - The first call on each device looks up the array's device address (one
+ *     cudaGetSymbolAddress); make that first call before any stream capture.
+ *   - All calls on a device share the one array, which keeps the last call's
+ *     contents; each call clears the counters it needs on `stream`.  Calls that
+ *     overlap on the GPU (other streams, or unordered launches) race on it.
+ * Errors as darb_lstm_step, plus DARB_ERR_UNSUPPORTED for the size limit.
+ */
+DARB_API darb_status_t darb_lstm_step_noalloc(darb_handle_t h, int64_t I, int64_t H, int64_t B,
+                                              const float *x, const float *h_prev, const float *c_prev,
+                                              const float *bias, float *h_out, float *c_out,
+                                              cudaStream_t stream);
+
 /* Size the handle's RNN step scratch for batches up to max_batch now, so that
  * later step calls allocate nothing (e.g. before capturing them in a CUDA
  * graph).  Synchronises the device.  Errors: INVALID_ARG, OOM, CUDA.          */

@@ -681,3 +681,24 @@ darb_status_t darb_destroy(darb_handle_t h) {
 }
 
 }  // extern "C"
+
+namespace darb {
+
+darb_status_t lstm_step_view(darb_handle_t h, int64_t I, int64_t H, int64_t B, const float *x,
+                             const float *h_prev, const float *c_prev, const float *bias,
+                             const float *h_out, const float *c_out, Format *f) {
+    darb_status_t st = check_step(h, I, H, B, 4, x, h_prev);
+    if (st != DARB_OK) return st;
+    if (c_prev == nullptr || h_out == nullptr || c_out == nullptr || f == nullptr) return DARB_ERR_INVALID_ARG;
+    const size_t hb = static_cast<size_t>(H * B) * 4;
+    const void *ins[4] = {x, h_prev, c_prev, bias};
+    const size_t inb[4] = {static_cast<size_t>(I * B) * 4, hb, hb, static_cast<size_t>(4 * H) * 4};
+    for (int i = 0; i < 4; ++i)
+        if (overlaps(h_out, hb, ins[i], inb[i]) || overlaps(c_out, hb, ins[i], inb[i]))
+            return DARB_ERR_INVALID_ARG;
+    if (overlaps(h_out, hb, c_out, hb)) return DARB_ERR_INVALID_ARG;
+    *f = format_of(h);
+    return DARB_OK;
+}
+
+}  // namespace darb

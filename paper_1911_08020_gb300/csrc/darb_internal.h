@@ -22,6 +22,8 @@
 #include <cstdint>
 #include <cuda_runtime.h>
 
+#include "darb.h"
+
 namespace darb {
 
 constexpr int kSlots = 32;   // rows per group
@@ -104,5 +106,11 @@ int rnn_batch_tile(int64_t B);
 
 // Streaming multiprocessors of the current device (cached).
 int sm_count();
+
+// The argument checks of darb_lstm_step and the handle's read-only view, for
+// an entry point that brings its own scratch.  Allocates nothing.
+darb_status_t lstm_step_view(darb_handle_t h, int64_t I, int64_t H, int64_t B, const float *x,
+                             const float *h_prev, const float *c_prev, const float *bias,
+                             const float *h_out, const float *c_out, Format *f);
 
 }  // namespace darb

@@ -56,6 +56,7 @@ def lib():
                 "darb_sync_status": [P, S],
                 "darb_spmm": [P, P, I64, I64, P, I64, S],
                 "darb_lstm_step": [P, I64, I64, I64, P, P, P, P, P, P, S],
+                "darb_lstm_step_noalloc": [P, I64, I64, I64, P, P, P, P, P, P, S],
                 "darb_gru_step": [P, I64, I64, I64, P, P, P, P, P, S],
                 "darb_rnn_reserve": [P, I64],
                 "darb_info": [P, P],
@@ -187,6 +188,18 @@ def darb_lstm_step(h: Handle, I: int, H: int, B: int, x, h_prev, c_prev, bias, h
         _require_cuda_f32(t, n)
     _check(lib().darb_lstm_step(h.ptr, I, H, B, _ptr(x), _ptr(h_prev), _ptr(c_prev), _ptr(bias),
                                 _ptr(h_out), _ptr(c_out), _stream(stream)), "darb_lstm_step")
+
+
+def darb_lstm_step_noalloc(h: Handle, I: int, H: int, B: int, x, h_prev, c_prev, bias, h_out, c_out,
+                           stream=None):
+    """darb_lstm_step with its scratch in the library's fixed 4 MiB array: no
+    allocation at call time (for callers that cannot let a library allocate)."""
+    for t, n in ((x, "x"), (h_prev, "h_prev"), (c_prev, "c_prev"), (bias, "bias"),
+                 (h_out, "h_out"), (c_out, "c_out")):
+        _require_cuda_f32(t, n)
+    _check(lib().darb_lstm_step_noalloc(h.ptr, I, H, B, _ptr(x), _ptr(h_prev), _ptr(c_prev),
+                                        _ptr(bias), _ptr(h_out), _ptr(c_out), _stream(stream)),
+           "darb_lstm_step_noalloc")
 
 
 def darb_gru_step(h: Handle, I: int, H: int, B: int, x, h_prev, b_ih, b_hh, h_out, stream=None):
