@@ -44,6 +44,9 @@ def parse_args():
     p.add_argument("--impl", choices=("darb", "reference"), default="darb")
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu", action="store_true")
+    p.add_argument("--no-rnn", action="store_true")
+    p.add_argument("--calls", default="",
+                   help="comma list restricting the step to some calls, e.g. fc6_spmm_b256 (profiling)")
     return p.parse_args()
 
 
@@ -55,6 +58,41 @@ def measured_peaks():
         return float(d["hbm_gbs"]), "measured"
     except (OSError, KeyError, ValueError):
         return FALLBACK_HBM_GBS, "fallback"
+
+
+def library_source_hash() -> str:
+    """sha1 over the library's CUDA sources: identifies the kernels a profile was taken on."""
+    import hashlib
+    csrc = os.path.join(ROOT, "paper_1911_08020_gb300", "csrc")
+    h = hashlib.sha1()
+    for name in sorted(os.listdir(csrc)):
+        if name.endswith((".cu", ".cuh", ".h")):
+            with open(os.path.join(csrc, name), "rb") as f:
+                h.update(name.encode() + b"\0" + f.read())
+    return h.hexdigest()[:12]
+
+
+def profiled_traffic(call: str):
+    """DRAM bytes per launch of `call` from the committed ncu summaries under
+    profiles/ (lines 'traffic: <call> <bytes> src=<hash>'), or None when no
+    summary was taken on the current kernels."""
+    pdir = os.path.join(ROOT, "profiles")
+    if not os.path.isdir(pdir):
+        return None
+    want = library_source_hash()
+    for name in sorted(os.listdir(pdir)):
+        if not name.endswith((".md", ".txt")):
+            continue
+        with open(os.path.join(pdir, name)) as f:
+            for ln in f:
+                parts = ln.strip().strip("`").split()
+                if len(parts) == 4 and parts[0] == "traffic:" and parts[1] == call and parts[3] == f"src={want}":
+                    return int(parts[2])
+    return None
+
+
+def call_name(kind, mi, b):
+    return ("fc6" if mi == 0 else "fc7") + ("_encode" if kind == "encode" else f"_spmm_b{b}")
 
 
 # ----------------------------------------------------------------------------- clocks
@@ -162,7 +200,7 @@ def encode_bytes(info):
 class Workload:
     """Rotating sets of device buffers for the FC6/FC7 step."""
 
-    def __init__(self, torch, darb, synth):
+    def __init__(self, torch, darb, synth, only=()):
         self.torch, self.darb = torch, darb
         wl = synth.WORKLOADS[WORKLOAD]
         dev = torch.device("cuda", torch.cuda.current_device())
@@ -197,6 +235,8 @@ class Workload:
         for b in BATCHES:
             for mi, mat in enumerate(self.mats):
                 self.calls.append(("spmm", mi, b, spmm_bytes(mat["info"], b)))
+        if only:
+            self.calls = [c for c in self.calls if call_name(*c[:3]) in only]
         self.step_bytes = sum(c[3] for c in self.calls)
 
     def launch(self, call, s, stream):
@@ -229,7 +269,8 @@ def run_gpu(args, world, rank, local):
 
     from paper_1911_08020_gb300 import darb, synth
     torch.cuda.set_device(local)
-    wl = Workload(torch, darb, synth)
+    only = tuple(c for c in args.calls.split(",") if c)
+    wl = Workload(torch, darb, synth, only)
     stream = torch.cuda.current_stream()
     sid = stream.cuda_stream
     ncalls = len(wl.calls)
@@ -274,25 +315,32 @@ def run_gpu(args, world, rank, local):
         per_call[i] = a.elapsed_time(b) / args.steps
     wl.check_encode()
     peak, peak_kind = measured_peaks()
+    clocks = clk.summary()
+    sm_mhz = (clocks or {}).get("sm_mhz") or 2070.0
+    nsm = torch.cuda.get_device_properties(torch.cuda.current_device()).multi_processor_count
+    # on-chip gather bound: every (kept weight, batch column) product reads its
+    # 4-byte activation from shared memory, at most 128 bytes/clock/SM
+    gather_peak = 128.0 * nsm * sm_mhz * 1e6 / 1e9   # GB/s
     parts = []
     for i, (kind, mi, b, nbytes) in enumerate(wl.calls):
-        name = ("fc6" if mi == 0 else "fc7") + ("_encode" if kind == "encode" else f"_spmm_b{b}")
-        gbs = nbytes / (per_call[i] * 1e-3) / 1e9
-        parts.append({"call": name, "bytes": int(nbytes), "us": round(per_call[i] * 1e3, 3),
-                      "gbs": round(gbs, 1), "hbm_frac": round(gbs / peak, 4),
-                      "gflops": round(2 * wl.mats[mi]["info"]["nnzb"] * b / (per_call[i] * 1e-3) / 1e9, 1)
-                      if kind == "spmm" else None})
-    # dominant kernel: the call kind/batch with the largest share of the step
-    kinds = {}
-    for p, i in zip(parts, range(ncalls)):
-        key = p["call"].split("_", 1)[1]
-        k = kinds.setdefault(key, [0.0, 0, 0])
-        k[0] += per_call[i]
-        k[1] += p["bytes"]
-        k[2] += 1
-    dom = max(kinds, key=lambda k: kinds[k][0])
-    dom_ms, dom_bytes, dom_n = kinds[dom]
-    achieved = dom_bytes / (dom_ms * 1e-3) / 1e9
+        name = call_name(kind, mi, b)
+        sec = per_call[i] * 1e-3
+        gbs = nbytes / sec / 1e9
+        part = {"call": name, "bytes": int(nbytes), "us": round(per_call[i] * 1e3, 3),
+                "gbs": round(gbs, 1), "hbm_frac": round(gbs / peak, 4)}
+        if kind == "spmm":
+            nnzb = wl.mats[mi]["info"]["nnzb"]
+            part["gflops"] = round(2 * nnzb * b / sec / 1e9, 1)
+            if b > 4:
+                part["gather_frac"] = round(nnzb * b * 4 / sec / 1e9 / gather_peak, 4)
+        parts.append(part)
+    # dominant kernel: the single call with the largest share of the step
+    di = int(np.argmax(per_call))
+    dom = parts[di]["call"]
+    dom_ms = float(per_call[di])
+    achieved = wl.calls[di][3] / (dom_ms * 1e-3) / 1e9
+    traffic = profiled_traffic(dom)
+    step_ms_sum = float(per_call.sum())
     value = world * wl.step_bytes / (ms_per_step * 1e-3) / 1e9
 
     result = {
@@ -307,18 +355,102 @@ def run_gpu(args, world, rank, local):
                    "pruning_ratio": [round(m["rows"] * m["cols"] / m["info"]["nnzb"], 2) for m in wl.mats],
                    "l2": f"inputs rotate over {NSETS} buffer sets (>4x L2), every call reads cold HBM",
                    "parallelism": f"replicas{world}"},
-        "roofline": {"bound": "hbm", "kernel": dom, "achieved": round(achieved, 1), "peak": peak,
-                     "peak_kind": peak_kind, "unit": "GB/s", "frac": round(achieved / peak, 4),
-                     "traffic": None},
+        "roofline": {"bound": "hbm", "kernel": dom, "achieved": round(achieved, 1),
+                     "peak": peak, "peak_kind": peak_kind, "unit": "GB/s", "frac": round(achieved / peak, 4),
+                     "frac_of_nominal_8000": round(achieved / 8000.0, 4),
+                     "share_of_step": round(dom_ms / step_ms_sum, 3) if step_ms_sum > 0 else None,
+                     "traffic": traffic,
+                     "note": "achieved = algorithmic bytes per launch (values + offsets + row metadata + X + Y,"
+                             " or dense W + encoding for encode) / mean launch time; for batch > 4 the"
+                             " on-chip activation gather, not HBM, binds (parts[].gather_frac)"},
+        "gather_peak_gbs": round(gather_peak, 1),
         "parts": parts,
         "parts_note": "per call: K launches of that call alone, back to back on rotating cold buffers",
         "gpu_launches": ncalls * args.steps,
-        "clocks": clk.summary(),
+        "clocks": clocks,
     }
+    if not args.no_rnn and not only:
+        result["rnn"] = run_rnn(torch, darb, synth, peak)
     if not args.no_e2e:
         result["e2e"] = run_e2e(args, wl, torch, darb)
     wl.close()
     return result
+
+
+def run_rnn(torch, darb, synth, peak, reps=3):
+    """The fused RNN steps on their workloads: whole sequences, device-timed.
+
+    The gate matrices (at most ~3 MB encoded) stay in L2 from one step to the
+    next, so the per-step GB/s here are L2-served, not HBM."""
+    dev = torch.device("cuda", torch.cuda.current_device())
+    out = {}
+
+    def seq_time(run):
+        run()
+        torch.cuda.synchronize()
+        times = []
+        for _ in range(reps):
+            a = torch.cuda.Event(enable_timing=True)
+            b = torch.cuda.Event(enable_timing=True)
+            a.record()
+            run()
+            b.record()
+            torch.cuda.synchronize()
+            times.append(a.elapsed_time(b))
+        return statistics.median(times)
+
+    def dev_matrix(wl, i):
+        _, stored, m = synth.matrix(wl, i)
+        if wl.dtype == "bf16":
+            W = torch.from_numpy(stored.view(np.int16)).to(dev).view(torch.bfloat16)
+        else:
+            W = torch.from_numpy(stored).to(dev)
+        h = darb.darb_encode(W, m)
+        return h, darb.darb_info(h)
+
+    def step_bytes(info, I, H, B, cell):
+        io = (I + H) * B * 4 + (2 if cell == "lstm" else 1) * H * B * 4   # inputs + outputs
+        io += H * B * 4 if cell == "lstm" else 0                           # c_prev
+        bias = info["rows"] * 4 * (1 if cell == "lstm" else 2)
+        return info["value_bytes"] + info["offset_bytes"] + info["meta_bytes"] + io + bias
+
+    for name in ("lstm_1024", "lstm_lm_1500", "gru_1024"):
+        wl = synth.WORKLOADS[name]
+        I, H = wl.input_size, wl.hidden
+        hs = [dev_matrix(wl, i) for i in range(wl.layers)]
+        for B in wl.batches:
+            xs = torch.from_numpy(np.ascontiguousarray(synth.rnn_inputs(wl, B, wl.steps))).to(dev)
+            hbuf = [torch.zeros((wl.layers, H, B), device=dev) for _ in range(2)]
+            cbuf = [torch.zeros((wl.layers, H, B), device=dev) for _ in range(2)]
+            bias = [torch.from_numpy(synth.bias(h[1]["rows"], seed=wl.seed + li)).to(dev) for li, h in enumerate(hs)]
+            bias2 = [torch.from_numpy(synth.bias(h[1]["rows"], seed=wl.seed + 7 + li)).to(dev) for li, h in enumerate(hs)]
+            for h, _ in hs:
+                darb.darb_rnn_reserve(h, B)
+
+            def run():
+                for t in range(wl.steps):
+                    src, dst = t % 2, (t + 1) % 2
+                    inp = xs[t]
+                    for li, (h, _) in enumerate(hs):
+                        if wl.kind == "lstm":
+                            darb.darb_lstm_step(h, I, H, B, inp, hbuf[src][li], cbuf[src][li], bias[li],
+                                                hbuf[dst][li], cbuf[dst][li])
+                        else:
+                            darb.darb_gru_step(h, I, H, B, inp, hbuf[src][li], bias[li], bias2[li],
+                                               hbuf[dst][li])
+                        inp = hbuf[dst][li]
+
+            ms = seq_time(run)
+            nsteps = wl.steps * wl.layers
+            us = ms * 1e3 / nsteps
+            nbytes = sum(step_bytes(info, I, H, B, wl.kind) for _, info in hs) / wl.layers
+            out[f"{name}_b{B}"] = {"cell": wl.kind, "layers": wl.layers, "timesteps": wl.steps, "batch": B,
+                                   "us_per_cell_step": round(us, 2), "gbs_l2_served": round(nbytes / (us * 1e-6) / 1e9, 1),
+                                   "gflops": round(2 * sum(i["nnzb"] for _, i in hs) / wl.layers * B / (us * 1e-6) / 1e9, 1),
+                                   "sequence_ms": round(ms, 3)}
+        for h, _ in hs:
+            darb.darb_destroy(h)
+    return out
 
 
 def run_e2e(args, wl, torch, darb):
@@ -389,7 +521,7 @@ def oracle_sample(budget_s: float = 12.0):
         total_bytes += (rows * cols * 2 + vb + ob + meta) + sum(
             vb + ob + meta + cols * b * 4 + rows * b * 4 for b in (1, 16))
         reps += 1
-        if reps >= 50:
+        if reps >= 2000:
             break
     sample = f"FC7 4096x4096 bf16: oracle encode + darb_spmm at batch 1 and 16, x{reps}"
     return total_bytes / total_s / 1e9, total_s, cores, sample
