@@ -516,7 +516,7 @@ darb_status_t darb_lstm_step(darb_handle_t h, int64_t I, int64_t H, int64_t B, c
     if (st != DARB_OK) return st;
     darb::RnnScratch sc{h->d_gates, h->d_counters};
     return cuda_status(darb::launch_lstm_step(format_of(h), I, H, B, x, h_prev, c_prev, bias,
-                                              h_out, c_out, sc, stream));
+                                              h_out, c_out, sc, stream, early_ok(h, stream)));
 }
 
 darb_status_t darb_gru_step(darb_handle_t h, int64_t I, int64_t H, int64_t B, const float *x,
@@ -535,7 +535,7 @@ darb_status_t darb_gru_step(darb_handle_t h, int64_t I, int64_t H, int64_t B, co
     if (st != DARB_OK) return st;
     darb::RnnScratch sc{h->d_gates, h->d_counters};
     return cuda_status(darb::launch_gru_step(format_of(h), I, H, B, x, h_prev, b_ih, b_hh, h_out,
-                                             sc, stream));
+                                             sc, stream, early_ok(h, stream)));
 }
 
 darb_status_t darb_info(darb_handle_t h, darb_info_t *info) {

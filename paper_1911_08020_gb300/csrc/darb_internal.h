@@ -93,13 +93,20 @@ cudaError_t launch_spmm_batch(const Format &f, const float *X, int64_t ldx, int6
 cudaError_t launch_spmm(const Format &f, const float *X, int64_t ldx, int64_t batch, float *Y,
                         int64_t ldy, bool early, cudaStream_t stream);
 
+// `early` as for launch_spmm (the handle's values may be read before the
+// previous kernel on the stream finishes).
 cudaError_t launch_lstm_step(const Format &f, int64_t I, int64_t H, int64_t B, const float *x,
                              const float *h_prev, const float *c_prev, const float *bias,
-                             float *h_out, float *c_out, RnnScratch s, cudaStream_t stream);
+                             float *h_out, float *c_out, RnnScratch s, cudaStream_t stream,
+                             bool early = false);
 
 cudaError_t launch_gru_step(const Format &f, int64_t I, int64_t H, int64_t B, const float *x,
                             const float *h_prev, const float *b_ih, const float *b_hh,
-                            float *h_out, RnnScratch s, cudaStream_t stream);
+                            float *h_out, RnnScratch s, cudaStream_t stream, bool early = false);
+
+struct RnnArgs;
+// Batch > 4 RNN steps (rnn_batch.cu); mode is kModeLstm or kModeGru.
+cudaError_t launch_rnn_batch(const Format &f, const RnnArgs &ra, int mode, bool early, cudaStream_t stream);
 
 // Batch-tile width the RNN step kernels use for a batch of B (sizes the counters).
 int rnn_batch_tile(int64_t B);
