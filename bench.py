@@ -45,6 +45,8 @@ def parse_args():
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu", action="store_true")
     p.add_argument("--no-rnn", action="store_true")
+    p.add_argument("--cpu-seconds", type=float, default=30.0,
+                   help="CPU time budget of the oracle arm (--impl reference) over all its steps")
     p.add_argument("--calls", default="",
                    help="comma list restricting the step to some calls, e.g. fc6_spmm_b256 (profiling)")
     return p.parse_args()
@@ -565,7 +567,8 @@ def run_reference(args, world, rank):
     oracle.build()
     per_step = []
     for s in range(args.warmup + args.steps):
-        gbs, secs, cores, sample = oracle_sample(budget_s=max(0.5, 60.0 / max(1, args.steps + args.warmup)))
+        gbs, secs, cores, sample = oracle_sample(
+            budget_s=max(0.2, args.cpu_seconds / max(1, args.steps + args.warmup)))
         if s >= args.warmup:
             per_step.append(secs)
         last = (gbs, cores, sample)
