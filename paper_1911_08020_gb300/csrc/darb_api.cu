@@ -26,7 +26,7 @@ struct darb_handle_s {
     // host copy of the layout
     std::vector<Group> groups;
     std::vector<int32_t> rowmap, rowloc, row_m;
-    std::vector<int2> enc_tiles;   // (row, first block) of every encoder tile
+    std::vector<darb::EncTile> enc_tiles;   // every encoder tile, resolved
     std::vector<int2> sets;        // row sets of up to 1, 2, 4, 8 groups, concatenated
     int32_t nsets[4] = {0, 0, 0, 0};
     int64_t val_elems = 0, off_words = 0;
@@ -34,7 +34,7 @@ struct darb_handle_s {
     void *dmem = nullptr;
     size_t dbytes = 0;
     Group *d_groups = nullptr;
-    int2 *d_tiles = nullptr;
+    darb::EncTile *d_tiles = nullptr;
     int2 *d_sets = nullptr;
     int32_t *d_rowmap = nullptr, *d_rowloc = nullptr, *d_row_m = nullptr, *d_status = nullptr;
     void *d_vals = nullptr;
@@ -157,10 +157,23 @@ void build_layout(darb_handle_s *h, const int32_t *m) {
     }
     h->enc_tiles.clear();
     for (int64_t r = 0; r < rows; ++r) {
-        const int tb = darb::enc_tile_blocks(m[r]);
-        const int64_t n = ceil_div(cols, m[r]);
-        for (int64_t jt = 0; jt < n; jt += tb)
-            h->enc_tiles.push_back(make_int2(static_cast<int>(r), static_cast<int>(jt)));
+        const int32_t loc = h->rowloc[static_cast<size_t>(r)];
+        const Group &g = h->groups[static_cast<size_t>(loc / kSlots)];
+        const int64_t slot = loc % kSlots;
+        const int tb = darb::enc_tile_blocks(g.m);
+        for (int64_t jt = 0; jt < g.n; jt += tb) {
+            darb::EncTile t{};
+            const int64_t nb = std::min<int64_t>(tb, g.n - jt);
+            const int64_t rec = (jt / kChunk) * kSlots + slot;   // jt is a multiple of the chunk
+            t.row = static_cast<int32_t>(r);
+            t.c0 = static_cast<int32_t>(jt * g.m);
+            t.span = static_cast<int32_t>(std::min<int64_t>(cols, (jt + nb) * g.m) - jt * g.m);
+            t.m = static_cast<int16_t>(g.m);
+            t.nb = static_cast<int16_t>(nb);
+            t.val_base = g.val_off + rec * kChunk;
+            t.off_base = g.off_off + rec * (g.nib ? 1 : 2);
+            h->enc_tiles.push_back(t);
+        }
     }
 }
 
@@ -168,7 +181,7 @@ darb_status_t alloc_device(darb_handle_s *h) {
     const size_t esz = h->wtype == DARB_BF16 ? 2 : 4;
     size_t o = 0;
     const size_t o_groups = o; o = align_up(o + h->groups.size() * sizeof(Group), 256);
-    const size_t o_tiles = o;  o = align_up(o + h->enc_tiles.size() * sizeof(int2), 256);
+    const size_t o_tiles = o;  o = align_up(o + h->enc_tiles.size() * sizeof(darb::EncTile), 256);
     const size_t o_sets = o;   o = align_up(o + h->sets.size() * sizeof(int2), 256);
     const size_t o_rowmap = o; o = align_up(o + h->rowmap.size() * 4, 256);
     const size_t o_rowloc = o; o = align_up(o + h->rowloc.size() * 4, 256);
@@ -183,7 +196,7 @@ darb_status_t alloc_device(darb_handle_s *h) {
     h->dmem = p;
     h->dbytes = o;
     h->d_groups = reinterpret_cast<Group *>(b + o_groups);
-    h->d_tiles = reinterpret_cast<int2 *>(b + o_tiles);
+    h->d_tiles = reinterpret_cast<darb::EncTile *>(b + o_tiles);
     h->d_sets = reinterpret_cast<int2 *>(b + o_sets);
     h->d_rowmap = reinterpret_cast<int32_t *>(b + o_rowmap);
     h->d_rowloc = reinterpret_cast<int32_t *>(b + o_rowloc);
@@ -200,7 +213,7 @@ darb_status_t upload_layout(darb_handle_s *h, cudaStream_t stream) {
         e = cudaMemcpyAsync(h->d_groups, h->groups.data(), h->groups.size() * sizeof(Group),
                             cudaMemcpyHostToDevice, stream);
     if (e == cudaSuccess)
-        e = cudaMemcpyAsync(h->d_tiles, h->enc_tiles.data(), h->enc_tiles.size() * sizeof(int2),
+        e = cudaMemcpyAsync(h->d_tiles, h->enc_tiles.data(), h->enc_tiles.size() * sizeof(darb::EncTile),
                             cudaMemcpyHostToDevice, stream);
     if (e == cudaSuccess)
         e = cudaMemcpyAsync(h->d_sets, h->sets.data(), h->sets.size() * sizeof(int2),
@@ -254,9 +267,6 @@ Format format_of(const darb_handle_s *h) {
 
 darb::EncodeTarget target_of(darb_handle_s *h) {
     darb::EncodeTarget t{};
-    t.groups = h->d_groups;
-    t.rowloc = h->d_rowloc;
-    t.row_m = h->d_row_m;
     t.tiles = h->d_tiles;
     t.ntiles = static_cast<int32_t>(h->enc_tiles.size());
     t.vals = h->d_vals;

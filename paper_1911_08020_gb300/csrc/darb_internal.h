@@ -62,12 +62,23 @@ struct Format {
     int64_t rows, cols;
 };
 
+// One encoder tile (a row, or a run of whole blocks of a long row), resolved
+// on the host: where it sits in W and where its blocks go in the format, so
+// that the encoder gets a tile from one 32-byte load instead of a chain of
+// dependent lookups (tile -> row -> slot -> group).
+struct __align__(16) EncTile {
+    int32_t row;       // matrix row
+    int32_t c0;        // first column, (first block) * m
+    int32_t span;      // columns of W in the tile (the row's last tile may stop short)
+    int16_t m;         // the row's block size
+    int16_t nb;        // blocks in the tile, a multiple of the chunk except at the row's end
+    int64_t val_base;  // value index of the tile's first block in the row's slot
+    int64_t off_base;  // offs word index of the tile's first record (one word if m <= 16, else two)
+};
+
 // Writable view used by the encoder.
 struct EncodeTarget {
-    const Group *groups;
-    const int32_t *rowloc;
-    const int32_t *row_m;
-    const int2 *tiles;       // (row, first block) of every encoder tile, row-major
+    const EncTile *tiles;    // every encoder tile, row-major
     int32_t ntiles;
     void *vals;
     uint32_t *offs;

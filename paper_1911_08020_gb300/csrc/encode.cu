@@ -4,7 +4,9 @@
 // into blocks of m_r columns, keep the weight of largest magnitude in each
 // block (lowest column on a tie), store its value and its offset in the block.
 //
-// The work is a list of tiles (a row, or a run of whole blocks of a long row).
+// The work is a list of tiles (a row, or a run of whole blocks of a long row),
+// each resolved on the host into a 32-byte descriptor (position in W, block
+// size, destination in the format), so that a tile costs one load to find.
 // A persistent grid (two or three CTAs per SM) walks the list; each CTA keeps
 // the bulk (TMA) copies of its next tiles in flight in a ring of shared-memory
 // buffers while it scans the current one, so the HBM read of W -- the only
@@ -21,7 +23,8 @@
 // t*m mod 32 then start 1..2^a-1 words apart, so every scan step is
 // conflict-free for any m.  Because the order is rotated, ties are resolved
 // explicitly by the smaller offset: for bf16, key = |w| << 16 | (0xFFFF - offset)
-// and one unsigned max per element does both; fp32 compares (|w|, offset).
+// and one unsigned max per element does both (two per 32-bit word when m is
+// even, the rotation then counted in words); fp32 compares (|w|, offset).
 #include "darb_internal.h"
 #include "launch.cuh"
 #include "tma.cuh"
@@ -40,37 +43,41 @@ __host__ __device__ constexpr int raw_bytes() { return kEncTileElems * (BF16 ? 2
 template <bool BF16>
 __host__ __device__ constexpr int enc_stages() { return BF16 ? 3 : 2; }
 
+// shared memory: [0, 32) one mbarrier per stage, [32, 128) the descriptor of
+// the tile in each stage, then the stages' raw buffers
 template <bool BF16>
 __host__ __device__ constexpr size_t encode_smem() {
     return 128 + size_t(enc_stages<BF16>()) * raw_bytes<BF16>();
 }
+static_assert(enc_stages<true>() * sizeof(EncTile) <= 96 && enc_stages<false>() * sizeof(EncTile) <= 96,
+              "tile descriptors must fit in the shared-memory header");
 
+__device__ __forceinline__ EncTile load_tile(const EncTile *p) {
+    union {
+        int4 v[2];
+        EncTile t;
+    } u;
+    const int4 *q = reinterpret_cast<const int4 *>(p);
+    u.v[0] = __ldg(q);
+    u.v[1] = __ldg(q + 1);
+    return u.t;
+}
+
+// Where a tile sits in W and which of its bytes the bulk copy moves.
 struct TileGeo {
-    int64_t r;
-    int jt, nb, m, span;     // first block, blocks, block size, columns
-    const char *gaddr;       // first byte of the tile in W
-    int off0;                // gaddr - (gaddr rounded down to 16 bytes)
-    int blo, bhi;            // bulk-copied byte range, relative to the rounded-down address
+    const char *gaddr;   // first byte of the tile in W
+    int off0;            // gaddr - (gaddr rounded down to 16 bytes)
+    int blo, bhi;        // bulk-copied byte range, relative to the rounded-down address
 };
 
 template <bool BF16>
-__device__ __forceinline__ TileGeo tile_geo(const EncodeTarget &t, const void *W, int64_t ldw, int i) {
+__device__ __forceinline__ TileGeo tile_geo(const EncTile &d, const void *W, int64_t ldw) {
     constexpr int kEsz = BF16 ? 2 : 4;
     TileGeo g;
-    const int2 tl = t.tiles[i];
-    g.r = tl.x;
-    g.jt = tl.y;
-    g.m = t.row_m[g.r];
-    const int n = t.groups[t.rowloc[g.r] / kSlots].n;
-    g.nb = min(enc_tile_blocks(g.m), n - g.jt);
-    const int64_t c0 = int64_t(g.jt) * g.m;
-    const int64_t c1 = min(t.cols, c0 + int64_t(g.nb) * g.m);
-    g.span = static_cast<int>(c1 - c0);
-    g.gaddr = static_cast<const char *>(W) + (g.r * ldw + c0) * kEsz;
-    const uintptr_t a = reinterpret_cast<uintptr_t>(g.gaddr);
-    g.off0 = static_cast<int>(a & 15);
+    g.gaddr = static_cast<const char *>(W) + (int64_t(d.row) * ldw + d.c0) * kEsz;
+    g.off0 = static_cast<int>(reinterpret_cast<uintptr_t>(g.gaddr) & 15);
     g.blo = (g.off0 + 15) & ~15;
-    g.bhi = (g.off0 + g.span * kEsz) & ~15;
+    g.bhi = (g.off0 + d.span * kEsz) & ~15;
     if (g.bhi < g.blo) g.bhi = g.blo;
     return g;
 }
@@ -82,8 +89,9 @@ encode_kernel(EncodeTarget t, const void *W, int64_t ldw, int32_t *status) {
     constexpr int kStages = enc_stages<BF16>();
     using elem_t = typename std::conditional<BF16, uint16_t, uint32_t>::type;
     extern __shared__ __align__(128) unsigned char sm[];
-    uint64_t *bar = reinterpret_cast<uint64_t *>(sm);   // one per stage
-    unsigned char *const raw0 = sm + 128;               // stage s at raw0 + s * raw_bytes
+    uint64_t *bar = reinterpret_cast<uint64_t *>(sm);        // one per stage
+    EncTile *s_tile = reinterpret_cast<EncTile *>(sm + 32);   // the tile in each stage
+    unsigned char *const raw0 = sm + 128;                    // stage s at raw0 + s * raw_bytes
     const int tid = threadIdx.x, lane = tid & 31;
 
     pdl_launch_dependents();
@@ -94,8 +102,10 @@ encode_kernel(EncodeTarget t, const void *W, int64_t ldw, int32_t *status) {
     __syncthreads();
     pdl_wait_previous();   // W may come from the previous kernel; outputs may still be read by it
 
-    auto issue = [&](int i, int s) {
-        const TileGeo g = tile_geo<BF16>(t, W, ldw, i);
+    // thread 0 only: record tile d in stage s and start its bulk copy
+    auto issue = [&](const EncTile &d, int s) {
+        s_tile[s] = d;
+        const TileGeo g = tile_geo<BF16>(d, W, ldw);
         const uint32_t bytes = uint32_t(g.bhi - g.blo);
         mbar_arrive_expect_tx(&bar[s], bytes);
         if (bytes > 0) bulk_g2s(raw0 + s * raw_bytes<BF16>() + g.blo, g.gaddr - g.off0 + g.blo, bytes, &bar[s]);
@@ -104,50 +114,74 @@ encode_kernel(EncodeTarget t, const void *W, int64_t ldw, int32_t *status) {
     bool nan = false, ok = true;
     uint32_t phases = 0u;   // bit s: parity of stage s's next phase
     int it = 0;
-    if (tid == 0)
+    EncTile next{};         // thread 0: descriptor of the next tile to issue, loaded one iteration early
+    if (tid == 0) {
         for (int k = 0; k < kStages - 1; ++k) {
             const int i = blockIdx.x + k * gridDim.x;
-            if (i < t.ntiles) issue(i, k);
+            if (i < t.ntiles) issue(load_tile(t.tiles + i), k);
         }
+        const int i = blockIdx.x + (kStages - 1) * gridDim.x;
+        if (i < t.ntiles) next = load_tile(t.tiles + i);
+    }
     for (int i = blockIdx.x; i < t.ntiles; i += gridDim.x, ++it) {
         const int s = it % kStages;
-        const TileGeo g = tile_geo<BF16>(t, W, ldw, i);
         const int iahead = i + (kStages - 1) * gridDim.x;
         if (iahead < t.ntiles && tid == 0) {
             fence_proxy_async_smem();   // earlier generic accesses to that stage come first
-            issue(iahead, (it + kStages - 1) % kStages);
+            issue(next, (it + kStages - 1) % kStages);
+            if (iahead + int(gridDim.x) < t.ntiles) next = load_tile(t.tiles + iahead + gridDim.x);
         }
         ok = __syncthreads_and(mbar_wait(&bar[s], (phases >> s) & 1u));
         phases ^= 1u << s;
         if (!ok) break;
-        const int m = g.m;
-        const int padded = g.nb * m;   // <= kEncTileElems
+        const EncTile d = s_tile[s];
+        const TileGeo g = tile_geo<BF16>(d, W, ldw);
+        const int m = d.m, nb = d.nb;
+        const bool nib = m <= 16;
+        const int padded = nb * m;   // <= kEncTileElems
         // element c of the tile sits at word c of `e`; fill the bytes the bulk
         // copy did not cover (unaligned head and tail) and zero the padding
         elem_t *e = reinterpret_cast<elem_t *>(raw0 + s * raw_bytes<BF16>() + g.off0);
-        const elem_t *src = reinterpret_cast<const elem_t *>(g.gaddr);
         const int ehead = (g.blo - g.off0) / kEsz, etail = (g.bhi - g.off0) / kEsz;
-        for (int c = tid; c < ehead && c < padded; c += kEncThreads) e[c] = c < g.span ? __ldg(src + c) : elem_t(0);
-        for (int c = etail + tid; c < padded; c += kEncThreads) e[c] = c < g.span ? __ldg(src + c) : elem_t(0);
-        __syncthreads();
-        // ---- one block per thread
-        const int loc = t.rowloc[g.r];
-        const Group grp = t.groups[loc / kSlots];
-        const int slot = loc % kSlots;
+        if (ehead > 0 || etail < padded) {   // the same for every thread
+            const elem_t *src = reinterpret_cast<const elem_t *>(g.gaddr);
+            for (int c = tid; c < ehead && c < padded; c += kEncThreads) e[c] = c < d.span ? __ldg(src + c) : elem_t(0);
+            for (int c = etail + tid; c < padded; c += kEncThreads) e[c] = c < d.span ? __ldg(src + c) : elem_t(0);
+            __syncthreads();
+        }
+        // ---- general path: one block per thread
         const int a = min(__ffs(m) - 1, 5);
         const int rot = (lane << a) >> 5;
-        for (int base = 0; base < g.nb; base += kEncThreads) {
+        // bf16 with an even block size and a 4-byte aligned tile: scan two
+        // elements per 32-bit word, rotating in word units (m/2 words per block)
+        const bool pairs = BF16 && (m % 2 == 0) && (g.off0 % 4 == 0);
+        const int mw = m >> 1;
+        const int aw = mw > 0 ? min(__ffs(mw) - 1, 5) : 0;
+        const int rotw = (lane << aw) >> 5;
+        for (int base = 0; base < nb; base += kEncThreads) {
             const int jj = base + tid;
-            const int j = g.jt + jj;
             uint32_t best_o = 0;
-            if (jj < g.nb) {
+            if (jj < nb) {
                 const elem_t *blk = e + jj * m;
                 int o = rot;
                 if constexpr (BF16) {
                     uint32_t best = 0;
-                    for (int k = 0; k < m; ++k) {
-                        best = max(best, ((uint32_t(blk[o]) & 0x7FFFu) << 16) | (0xFFFFu - uint32_t(o)));
-                        o = (o + 1 == m) ? 0 : o + 1;
+                    if (pairs) {
+                        const uint32_t *wblk = reinterpret_cast<const uint32_t *>(blk);
+                        int qw = rotw;
+#pragma unroll 2
+                        for (int k = 0; k < mw; ++k) {
+                            const uint32_t w = wblk[qw];
+                            const uint32_t i0 = 0xFFFFu - 2u * uint32_t(qw);   // key of element 2*qw
+                            best = max(best, ((w << 16) & 0x7FFF0000u) | i0);
+                            best = max(best, (w & 0x7FFF0000u) | (i0 - 1u));
+                            qw = (qw + 1 == mw) ? 0 : qw + 1;
+                        }
+                    } else {
+                        for (int k = 0; k < m; ++k) {
+                            best = max(best, ((uint32_t(blk[o]) & 0x7FFFu) << 16) | (0xFFFFu - uint32_t(o)));
+                            o = (o + 1 == m) ? 0 : o + 1;
+                        }
                     }
                     best_o = 0xFFFFu - (best & 0xFFFFu);
                     nan |= (best >> 16) > 0x7F80u;
@@ -164,28 +198,29 @@ encode_kernel(EncodeTarget t, const void *W, int64_t ldw, int32_t *status) {
                     }
                     nan |= best_a > 0x7F800000u;
                 }
-                const int64_t vi = grp.val_off + (int64_t(j / kChunk) * kSlots + slot) * kChunk + (j % kChunk);
-                static_cast<elem_t *>(t.vals)[vi] = blk[best_o];
+                static_cast<elem_t *>(t.vals)[d.val_base + int64_t(jj / kChunk) * (kSlots * kChunk) + jj % kChunk] =
+                    blk[best_o];
             }
             // pack the 8 offsets of a chunk: lanes 8q..8q+7 hold blocks 8c..8c+7
-            const int q = j % kChunk;
+            // (tiles start on a chunk boundary, so block jj is at position jj % 8)
+            const int q = jj % kChunk;
             uint32_t lo_w, hi_w;
-            if (grp.nib) {
-                lo_w = (jj < g.nb) ? (best_o << (4 * q)) : 0u;
+            if (nib) {
+                lo_w = (jj < nb) ? (best_o << (4 * q)) : 0u;
                 hi_w = 0u;
             } else {
-                lo_w = (jj < g.nb && q < 4) ? (best_o << (8 * q)) : 0u;
-                hi_w = (jj < g.nb && q >= 4) ? (best_o << (8 * (q - 4))) : 0u;
+                lo_w = (jj < nb && q < 4) ? (best_o << (8 * q)) : 0u;
+                hi_w = (jj < nb && q >= 4) ? (best_o << (8 * (q - 4))) : 0u;
             }
 #pragma unroll
-            for (int d = 1; d < kChunk; d <<= 1) {
-                lo_w |= __shfl_xor_sync(0xFFFFFFFFu, lo_w, d);
-                hi_w |= __shfl_xor_sync(0xFFFFFFFFu, hi_w, d);
+            for (int dd = 1; dd < kChunk; dd <<= 1) {
+                lo_w |= __shfl_xor_sync(0xFFFFFFFFu, lo_w, dd);
+                hi_w |= __shfl_xor_sync(0xFFFFFFFFu, hi_w, dd);
             }
-            if (q == 0 && jj < g.nb) {
-                const int64_t rec = int64_t(j / kChunk) * kSlots + slot;
-                if (grp.nib) t.offs[grp.off_off + rec] = lo_w;
-                else reinterpret_cast<uint2 *>(t.offs + grp.off_off)[rec] = make_uint2(lo_w, hi_w);
+            if (q == 0 && jj < nb) {
+                const int64_t c = jj / kChunk;
+                if (nib) t.offs[d.off_base + c * kSlots] = lo_w;
+                else reinterpret_cast<uint2 *>(t.offs + d.off_base)[c * kSlots] = make_uint2(lo_w, hi_w);
             }
         }
         __syncthreads();   // this stage is free for the copy issued next iteration

@@ -55,11 +55,14 @@ __device__ __forceinline__ void mbar_expect_tx(uint64_t *bar, uint32_t bytes) {
 }
 
 // Wait for the phase with the given parity to complete; false after the time
-// limit.  Each try_wait suspends the thread in hardware for up to ~10 us while
-// the phase is pending, so a waiting warp costs almost no issue slots.
+// limit.  Each try_wait may suspend the thread in hardware while the phase is
+// pending; between attempts the thread also sleeps with exponential back-off
+// (32 ns doubling to 512 ns) so that a warp waiting for a copy or for other
+// warps costs few issue slots.
 __device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity) {
     const uint32_t a = smem_addr(bar);
     unsigned long long t0 = 0;
+    unsigned sleep_ns = 32;
     while (true) {
         uint32_t done;
         asm volatile(
@@ -71,6 +74,8 @@ __device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity) {
         const unsigned long long now = global_timer_ns();
         if (t0 == 0) t0 = now;
         else if (now - t0 > kWaitLimitNs) return false;
+        __nanosleep(sleep_ns);
+        if (sleep_ns < 512) sleep_ns <<= 1;
     }
 }
 
