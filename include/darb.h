@@ -128,6 +128,29 @@ DARB_API darb_status_t darb_sync_status(darb_handle_t h, cudaStream_t stream);
 DARB_API darb_status_t darb_spmm(darb_handle_t h, const float *X, int64_t ldx, int64_t batch, float *Y,
                         int64_t ldy, cudaStream_t stream);
 
+/* Which kernels compute a product (the paper has no counterpart: these are two
+ * ways of evaluating the same sum on the GPU).                               */
+typedef enum {
+    DARB_PATH_AUTO = 0,          /* what darb_spmm does                              */
+    DARB_PATH_CUDA_CORES = 1,    /* gather-multiply-add on the CUDA cores (any weights) */
+    DARB_PATH_TENSOR_CORES = 2   /* densified tiles on the tensor cores (bf16 weights) */
+} darb_path_t;
+
+/*
+ * darb_spmm with the kernel family chosen by the caller.  DARB_PATH_AUTO uses
+ * the tensor cores for bf16 weights from 128 batch columns on when X allows
+ * it, else the CUDA cores.  The tensor-core path multiplies every activation
+ * of a stage by the densified tile, zeros included, with X split into two
+ * bf16 parts (x = hi + lo): |Y - exact| <= 2^-16 * sum |val * x| plus fp32
+ * rounding, a NaN or infinity in X may make rows NaN that do not select it,
+ * and |x| must stay below the largest bf16.  It needs bf16 weights, X 16-byte
+ * aligned and ldx a multiple of 4.
+ * Errors: as darb_spmm; DARB_ERR_INVALID_ARG for an unknown path;
+ * DARB_ERR_UNSUPPORTED if DARB_PATH_TENSOR_CORES cannot take the call.
+ */
+DARB_API darb_status_t darb_spmm_ex(darb_handle_t h, const float *X, int64_t ldx, int64_t batch, float *Y,
+                                    int64_t ldy, darb_path_t path, cudaStream_t stream);
+
 /*
  * One LSTM cell step whose gate matrix is the handle (rows = 4H, cols = I + H),
  * multiplied with the stacked input [x_t; h_{t-1}].  Gate rows [0,H) = i,

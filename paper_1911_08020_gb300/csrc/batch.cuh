@@ -419,20 +419,6 @@ batch_kernel(Format f, const int2 *__restrict__ sets, const float *__restrict__ 
     if (ksc > 1) cluster.sync();
 }
 
-inline PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
-    static PFN_cuTensorMapEncodeTiled_v12000 fn = [] {
-        void *p = nullptr;
-        cudaDriverEntryPointQueryResult q;
-        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) != cudaSuccess ||
-            q != cudaDriverEntryPointSuccess) {
-            cudaGetLastError();
-            return static_cast<PFN_cuTensorMapEncodeTiled_v12000>(nullptr);
-        }
-        return reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
-    }();
-    return fn;
-}
-
 // Tensor map over a rows x `batch` fp32 matrix (row pitch ld floats) with a
 // boxr x bt box; false if it cannot be described (alignment).
 inline bool make_map(CUtensorMap *map, const float *A, int64_t ld, int64_t batch, int64_t rows, int bt,

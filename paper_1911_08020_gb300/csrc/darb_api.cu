@@ -476,6 +476,13 @@ darb_status_t darb_sync_status(darb_handle_t h, cudaStream_t stream) {
 
 darb_status_t darb_spmm(darb_handle_t h, const float *X, int64_t ldx, int64_t batch, float *Y,
                         int64_t ldy, cudaStream_t stream) {
+    return darb_spmm_ex(h, X, ldx, batch, Y, ldy, DARB_PATH_AUTO, stream);
+}
+
+darb_status_t darb_spmm_ex(darb_handle_t h, const float *X, int64_t ldx, int64_t batch, float *Y,
+                           int64_t ldy, darb_path_t path, cudaStream_t stream) {
+    if (path != DARB_PATH_AUTO && path != DARB_PATH_CUDA_CORES && path != DARB_PATH_TENSOR_CORES)
+        return DARB_ERR_INVALID_ARG;
     if (!live(h) || X == nullptr || Y == nullptr || batch <= 0 || ldx < batch || ldy < batch)
         return DARB_ERR_INVALID_ARG;
     if (reinterpret_cast<uintptr_t>(X) % 4 != 0 || reinterpret_cast<uintptr_t>(Y) % 4 != 0)
@@ -484,8 +491,12 @@ darb_status_t darb_spmm(darb_handle_t h, const float *X, int64_t ldx, int64_t ba
     if (overlaps(X, static_cast<size_t>((h->cols - 1) * ldx + batch) * 4, Y,
                  static_cast<size_t>((h->rows - 1) * ldy + batch) * 4))
         return DARB_ERR_INVALID_ARG;
-    return cuda_status(
-        darb::launch_spmm(format_of(h), X, ldx, batch, Y, ldy, early_ok(h, stream), stream));
+    const cudaError_t e = darb::launch_spmm(format_of(h), X, ldx, batch, Y, ldy, early_ok(h, stream), path, stream);
+    if (e == cudaErrorNotSupported) {
+        cudaGetLastError();
+        return DARB_ERR_UNSUPPORTED;
+    }
+    return cuda_status(e);
 }
 
 darb_status_t darb_rnn_reserve(darb_handle_t h, int64_t max_batch) {

@@ -99,10 +99,21 @@ cudaError_t launch_encode(const EncodeTarget &t, const void *W, int64_t ldw, int
 cudaError_t launch_spmm_batch(const Format &f, const float *X, int64_t ldx, int64_t batch, float *Y,
                               int64_t ldy, bool early, cudaStream_t stream);
 
+// Tensor-core path (spmm_tc.cu): bf16 weights only; cudaErrorNotSupported
+// when the call does not fit it.
+cudaError_t launch_spmm_tc(const Format &f, const float *X, int64_t ldx, int64_t batch, float *Y,
+                           int64_t ldy, bool early, cudaStream_t stream);
+
+// Smallest batch that the automatic choice sends to the tensor cores: below
+// it the CUDA-core kernels are as fast (measured on the FC6/FC7 shapes).
+constexpr int64_t kTensorCoreMinBatch = 128;
+
 // `early`: the handle's data is known to be complete, so a kernel may start
 // reading it before the previous kernel on the stream has finished (PDL).
+// `path`: a darb_path_t.  cudaErrorNotSupported if DARB_PATH_TENSOR_CORES
+// was asked for a call the tensor-core kernel cannot take.
 cudaError_t launch_spmm(const Format &f, const float *X, int64_t ldx, int64_t batch, float *Y,
-                        int64_t ldy, bool early, cudaStream_t stream);
+                        int64_t ldy, bool early, int path, cudaStream_t stream);
 
 // `early` as for launch_spmm (the handle's values may be read before the
 // previous kernel on the stream finishes).

@@ -1,7 +1,10 @@
 // launch.cuh -- cudaLaunchKernelEx wrapper: thread-block clusters and
-// programmatic dependent launch (PDL) on the caller's stream.
+// programmatic dependent launch (PDL) on the caller's stream; the driver's
+// tensor-map encoder.
 #pragma once
 
+#include <cuda.h>
+#include <cudaTypedefs.h>
 #include <cuda_runtime.h>
 
 #include <utility>
@@ -41,6 +44,22 @@ cudaError_t allow_smem(void (*kernel)(KArgs...), size_t bytes) {
     if (bytes <= 48 * 1024) return cudaSuccess;
     return cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 static_cast<int>(bytes));
+}
+
+// cuTensorMapEncodeTiled from the driver (through the runtime, so that the
+// library does not link libcuda); nullptr if unavailable.
+inline PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = [] {
+        void *p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) != cudaSuccess ||
+            q != cudaDriverEntryPointSuccess) {
+            cudaGetLastError();
+            return static_cast<PFN_cuTensorMapEncodeTiled_v12000>(nullptr);
+        }
+        return reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+    }();
+    return fn;
 }
 
 }  // namespace darb

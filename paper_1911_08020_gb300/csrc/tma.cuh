@@ -56,10 +56,10 @@ __device__ __forceinline__ void mbar_expect_tx(uint64_t *bar, uint32_t bytes) {
 
 // Wait for the phase with the given parity to complete; false after the time
 // limit.  Each try_wait may suspend the thread in hardware while the phase is
-// pending; between attempts the thread also sleeps with exponential back-off
-// (32 ns doubling to 512 ns) so that a warp waiting for a copy or for other
-// warps costs few issue slots.
-__device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity) {
+// pending; with `backoff` the thread also sleeps between attempts (32 ns
+// doubling to 512 ns) so that a warp waiting long costs few issue slots,
+// without it the wait reacts as soon as the phase completes.
+__device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, bool backoff = true) {
     const uint32_t a = smem_addr(bar);
     unsigned long long t0 = 0;
     unsigned sleep_ns = 32;
@@ -74,8 +74,10 @@ __device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity) {
         const unsigned long long now = global_timer_ns();
         if (t0 == 0) t0 = now;
         else if (now - t0 > kWaitLimitNs) return false;
-        __nanosleep(sleep_ns);
-        if (sleep_ns < 512) sleep_ns <<= 1;
+        if (backoff) {
+            __nanosleep(sleep_ns);
+            if (sleep_ns < 512) sleep_ns <<= 1;
+        }
     }
 }
 

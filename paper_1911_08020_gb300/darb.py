@@ -19,6 +19,7 @@ LIB_PATH = os.path.join(_PKG, "libdarb.so")
 
 OK, ERR_INVALID_ARG, ERR_NONFINITE, ERR_OOM, ERR_CUDA, ERR_TIMEOUT, ERR_UNSUPPORTED = range(7)
 F32, BF16 = 0, 1
+PATH_AUTO, PATH_CUDA_CORES, PATH_TENSOR_CORES = 0, 1, 2
 MAX_BLOCK = 256
 
 _lock = threading.Lock()
@@ -55,6 +56,7 @@ def lib():
                 "darb_reencode": [P, P, I64, S],
                 "darb_sync_status": [P, S],
                 "darb_spmm": [P, P, I64, I64, P, I64, S],
+                "darb_spmm_ex": [P, P, I64, I64, P, I64, ctypes.c_int, S],
                 "darb_lstm_step": [P, I64, I64, I64, P, P, P, P, P, P, S],
                 "darb_lstm_step_noalloc": [P, I64, I64, I64, P, P, P, P, P, P, S],
                 "darb_gru_step": [P, I64, I64, I64, P, P, P, P, P, S],
@@ -165,6 +167,11 @@ def darb_sync_status(h: Handle, stream=None):
 
 def darb_spmm(h: Handle, X, Y=None, stream=None):
     """Y = W_darb X for X (cols x batch, CUDA float32); returns Y."""
+    return darb_spmm_ex(h, X, Y, PATH_AUTO, stream)
+
+
+def darb_spmm_ex(h: Handle, X, Y=None, path: int = PATH_AUTO, stream=None):
+    """darb_spmm with the kernel family chosen (PATH_AUTO, PATH_CUDA_CORES, PATH_TENSOR_CORES)."""
     import torch
     _require_cuda_f32(X, "X")
     if X.dim() == 1:
@@ -177,7 +184,11 @@ def darb_spmm(h: Handle, X, Y=None, stream=None):
     _require_cuda_f32(Y, "Y")
     ldx = X.stride(0) if X.shape[0] > 1 else batch
     ldy = Y.stride(0) if Y.shape[0] > 1 else batch
-    _check(lib().darb_spmm(h.ptr, _ptr(X), ldx, batch, _ptr(Y), ldy, _stream(stream)), "darb_spmm")
+    if path == PATH_AUTO:
+        _check(lib().darb_spmm(h.ptr, _ptr(X), ldx, batch, _ptr(Y), ldy, _stream(stream)), "darb_spmm")
+    else:
+        _check(lib().darb_spmm_ex(h.ptr, _ptr(X), ldx, batch, _ptr(Y), ldy, int(path), _stream(stream)),
+               "darb_spmm_ex")
     return Y
 
 
