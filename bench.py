@@ -34,6 +34,7 @@ BATCHES = (1, 16, 64, 256)
 METRIC = ("darb_spmm effective GB/s & % of HBM roofline at batch 1/16/64/256; encode GB/s")
 NSETS = 4
 FALLBACK_HBM_GBS = 6800.0
+FALLBACK_BF16_TFLOPS = 1900.0
 
 
 def parse_args():
@@ -60,6 +61,15 @@ def measured_peaks():
         return float(d["hbm_gbs"]), "measured"
     except (OSError, KeyError, ValueError):
         return FALLBACK_HBM_GBS, "fallback"
+
+
+def measured_bf16_tflops():
+    """Dense bf16 tensor peak (burst: a kernel timed alone), measured or fallback."""
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return float(json.load(f)["bf16_tflops"]), "measured"
+    except (OSError, KeyError, ValueError):
+        return FALLBACK_BF16_TFLOPS, "fallback"
 
 
 def library_source_hash() -> str:
@@ -210,6 +220,35 @@ def encode_bytes(info):
     return info["rows"] * info["cols"] * esz + info["value_bytes"] + info["offset_bytes"] + info["meta_bytes"]
 
 
+def tensor_flops(mat, batch):
+    """FLOPs of the densified product on the tensor cores: rows x cols x batch
+    multiply-adds for each of the two bf16 parts of X."""
+    return 2.0 * 2.0 * mat["rows"] * mat["cols"] * batch
+
+
+def roofline(wl, di, dom, dom_ms, achieved, peak, peak_kind, tpeak, tpeak_kind, traffic, step_ms_sum):
+    """Roofline of the dominant call: HBM bytes for the CUDA-core kernels and
+    the encoder, tensor FLOPs (bf16 peak) for the tensor-core product."""
+    kind, mi, b, nbytes = wl.calls[di]
+    share = round(dom_ms / step_ms_sum, 3) if step_ms_sum > 0 else None
+    if wl.paths[di][0] == "tensor":
+        tfl = tensor_flops(wl.mats[mi], b) / (dom_ms * 1e-3) / 1e12
+        return {"bound": "tensor", "kernel": dom, "achieved": round(tfl, 1), "peak": tpeak,
+                "peak_kind": tpeak_kind, "unit": "TFLOP/s", "frac": round(tfl / tpeak, 4),
+                "share_of_step": share, "traffic": traffic,
+                "hbm_gbs": round(achieved, 1), "hbm_frac": round(achieved / peak, 4),
+                "note": "achieved = 2 x 2 x rows x cols x batch (the densified product, once per bf16"
+                        " part of X) / mean call time (the split of X and the product kernel);"
+                        " peak = measured dense bf16 (burst)"}
+    return {"bound": "hbm", "kernel": dom, "achieved": round(achieved, 1),
+            "peak": peak, "peak_kind": peak_kind, "unit": "GB/s", "frac": round(achieved / peak, 4),
+            "frac_of_nominal_8000": round(achieved / 8000.0, 4), "share_of_step": share,
+            "traffic": traffic,
+            "note": "achieved = algorithmic bytes per launch (values + offsets + row metadata + X + Y,"
+                    " or dense W + encoding for encode) / mean launch time; for batch > 4 the"
+                    " on-chip activation gather, not HBM, binds (parts[].gather_frac)"}
+
+
 # ----------------------------------------------------------------------------- GPU arm
 class Workload:
     """Rotating sets of device buffers for the FC6/FC7 step."""
@@ -252,6 +291,15 @@ class Workload:
         if only:
             self.calls = [c for c in self.calls if call_name(*c[:3]) in only]
         self.step_bytes = sum(c[3] for c in self.calls)
+        # kernel family and launches of each call, as the library reports them
+        self.paths = []
+        for kind, mi, b, _ in self.calls:
+            if kind == "encode":
+                self.paths.append(("encode", 1))
+            else:
+                path, kernels = darb.darb_spmm_path(self.mats[mi]["h"], b)
+                self.paths.append(("tensor" if path == darb.PATH_TENSOR_CORES else "cuda", kernels))
+        self.step_launches = sum(k for _, k in self.paths)
 
     def launch(self, call, s, stream):
         kind, mi, b, _ = call
@@ -343,17 +391,24 @@ def run_gpu(args, world, rank, local):
     # on-chip gather bound: every (kept weight, batch column) product reads its
     # 4-byte activation from shared memory, at most 128 bytes/clock/SM
     gather_peak = 128.0 * nsm * sm_mhz * 1e6 / 1e9   # GB/s
+    tpeak, tpeak_kind = measured_bf16_tflops()
     parts = []
     for i, (kind, mi, b, nbytes) in enumerate(wl.calls):
         name = call_name(kind, mi, b)
         sec = per_call[i] * 1e-3
         gbs = nbytes / sec / 1e9
-        part = {"call": name, "bytes": int(nbytes), "us": round(per_call[i] * 1e3, 3),
-                "gbs": round(gbs, 1), "hbm_frac": round(gbs / peak, 4)}
+        path, kernels = wl.paths[i]
+        part = {"call": name, "path": path, "kernels": kernels, "bytes": int(nbytes),
+                "us": round(per_call[i] * 1e3, 3), "gbs": round(gbs, 1), "hbm_frac": round(gbs / peak, 4)}
         if kind == "spmm":
             nnzb = wl.mats[mi]["info"]["nnzb"]
             part["gflops"] = round(2 * nnzb * b / sec / 1e9, 1)
-            if b > 4:
+            if path == "tensor":
+                # the densified product the tensor cores execute: rows x cols x batch, twice (x = hi + lo)
+                tfl = tensor_flops(wl.mats[mi], b) / sec / 1e12
+                part["tensor_tflops"] = round(tfl, 1)
+                part["tensor_frac"] = round(tfl / tpeak, 4)
+            elif b > 4:
                 part["gather_frac"] = round(nnzb * b * 4 / sec / 1e9 / gather_peak, 4)
         parts.append(part)
     # dominant kernel: the single call with the largest share of the step
@@ -377,20 +432,14 @@ def run_gpu(args, world, rank, local):
                    "pruning_ratio": [round(m["rows"] * m["cols"] / m["info"]["nnzb"], 2) for m in wl.mats],
                    "l2": f"inputs rotate over {NSETS} buffer sets (>4x L2), every call reads cold HBM",
                    "parallelism": f"replicas{world}"},
-        "roofline": {"bound": "hbm", "kernel": dom, "achieved": round(achieved, 1),
-                     "peak": peak, "peak_kind": peak_kind, "unit": "GB/s", "frac": round(achieved / peak, 4),
-                     "frac_of_nominal_8000": round(achieved / 8000.0, 4),
-                     "share_of_step": round(dom_ms / step_ms_sum, 3) if step_ms_sum > 0 else None,
-                     "traffic": traffic,
-                     "note": "achieved = algorithmic bytes per launch (values + offsets + row metadata + X + Y,"
-                             " or dense W + encoding for encode) / mean launch time; for batch > 4 the"
-                             " on-chip activation gather, not HBM, binds (parts[].gather_frac)"},
+        "roofline": roofline(wl, di, dom, dom_ms, achieved, peak, peak_kind, tpeak, tpeak_kind, traffic,
+                             step_ms_sum),
         "gather_peak_gbs": round(gather_peak, 1),
         "parts": parts,
         "parts_note": "per call: K launches of that call alone, back to back on rotating cold buffers,"
                       " replayed from a CUDA graph",
         "timing": "CUDA-graph replay of whole steps (one graph per buffer set); CUDA events on the stream",
-        "gpu_launches": ncalls * args.steps,
+        "gpu_launches": wl.step_launches * args.steps,
         "clocks": clocks,
     }
     if not args.no_rnn and not only:

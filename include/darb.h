@@ -138,18 +138,27 @@ typedef enum {
 
 /*
  * darb_spmm with the kernel family chosen by the caller.  DARB_PATH_AUTO uses
- * the tensor cores for bf16 weights from 128 batch columns on when X allows
- * it, else the CUDA cores.  The tensor-core path multiplies every activation
+ * the tensor cores for bf16 weights from 33 batch columns on, else the CUDA
+ * cores.  The tensor-core path multiplies every activation
  * of a stage by the densified tile, zeros included, with X split into two
  * bf16 parts (x = hi + lo): |Y - exact| <= 2^-16 * sum |val * x| plus fp32
  * rounding, a NaN or infinity in X may make rows NaN that do not select it,
- * and |x| must stay below the largest bf16.  It needs bf16 weights, X 16-byte
- * aligned and ldx a multiple of 4.
+ * and |x| must stay below the largest bf16.  It needs bf16 weights, and it
+ * takes the split of X (4 bytes per element of X, batch rounded up to 8) from
+ * the device's stream-ordered memory pool on `stream` for the duration of the
+ * call (DARB_ERR_OOM if the pool cannot supply it); the CUDA-core path
+ * allocates nothing.
  * Errors: as darb_spmm; DARB_ERR_INVALID_ARG for an unknown path;
  * DARB_ERR_UNSUPPORTED if DARB_PATH_TENSOR_CORES cannot take the call.
  */
 DARB_API darb_status_t darb_spmm_ex(darb_handle_t h, const float *X, int64_t ldx, int64_t batch, float *Y,
                                     int64_t ldy, darb_path_t path, cudaStream_t stream);
+
+/* The kernel family darb_spmm takes for this handle and batch (*path), and
+ * how many kernels it launches per call (*kernels: 1 on the CUDA cores, 2 on
+ * the tensor cores, the split of X and the product).  Host only.
+ * Errors: DARB_ERR_INVALID_ARG (unknown handle, batch <= 0, null outputs). */
+DARB_API darb_status_t darb_spmm_path(darb_handle_t h, int64_t batch, darb_path_t *path, int32_t *kernels);
 
 /*
  * One LSTM cell step whose gate matrix is the handle (rows = 4H, cols = I + H),

@@ -496,7 +496,19 @@ darb_status_t darb_spmm_ex(darb_handle_t h, const float *X, int64_t ldx, int64_t
         cudaGetLastError();
         return DARB_ERR_UNSUPPORTED;
     }
+    if (e == cudaErrorMemoryAllocation) {
+        cudaGetLastError();
+        return DARB_ERR_OOM;
+    }
     return cuda_status(e);
+}
+
+darb_status_t darb_spmm_path(darb_handle_t h, int64_t batch, darb_path_t *path, int32_t *kernels) {
+    if (!live(h) || batch <= 0 || path == nullptr || kernels == nullptr) return DARB_ERR_INVALID_ARG;
+    const bool tensor = h->wtype == DARB_BF16 && batch >= darb::kTensorCoreMinBatch && batch <= kMaxBatch;
+    *path = tensor ? DARB_PATH_TENSOR_CORES : DARB_PATH_CUDA_CORES;
+    *kernels = tensor ? 2 : 1;
+    return DARB_OK;
 }
 
 darb_status_t darb_rnn_reserve(darb_handle_t h, int64_t max_batch) {

@@ -3,34 +3,40 @@
 //
 // Past a few dozen batch columns the CUDA-core product is bound by gathering
 // one activation operand from shared memory per (kept weight, column) pair.
-// This kernel instead densifies a slice of W_darb in shared memory and hands
+// This path instead densifies a slice of W_darb in shared memory and hands
 // the contraction to the tensor cores: the zeros cost m times the multiplies
 // of the sparse product, but a GB300 SM does them far faster than it can
 // gather.
 //
-// Work unit: 256 rows (eight consecutive 32-row groups, any block sizes) x
-// one batch tile of N = 32..256 columns x one cluster rank's share of the
-// columns of W.  The rank walks its share in stages of 32 columns:
-//  * a TMA warp copies the activation rows, X[k0 .. k0+32R) for the batch
-//    tile, into a ring of 32 KB fp32 staging slots, each holding R = 256/N
-//    stages (rows and columns past the ends read as zeros): about 64-96 KB of
-//    activations stay in flight per SM whatever the tile width;
-//  * four converter warps split the staged activations into two bf16 parts,
-//    x = hi + lo, written as two MN-major B tiles (128-byte swizzle);
-//  * eight producer warps (one thread per row; a warp is one 32-row group,
-//    so all its lanes share a block size and walk the blocks in lockstep)
-//    zero the row's 64 bytes of the stage and write the row's kept values
-//    that fall in it (bf16, exact) into two 128 x 32 A tiles (K-major,
-//    64-byte swizzle); for m >= 16 at most three blocks meet a stage and
-//    are decoded in straight-line code;
-//  * an MMA warp issues, per stage and 128-row half, A*B_hi + A*B_lo for two
-//    K=16 steps into that half's TMEM accumulator (128 lanes x N fp32
-//    columns) and releases the stage with tcgen05.commit.
-// At the end the ranks of a cluster add their partial accumulators: each rank
-// owns a slice of the rows, every rank stores its partial rows of that slice
-// into the owner's shared memory (distributed shared memory, no waiting on
-// remote loads), and the owner adds them in rank order (deterministic) and
-// writes its rows of Y.
+// Two kernels per call:
+//  * split_kernel writes X once as two bf16 arrays, x = hi + lo, into
+//    stream-ordered workspace (the tensor cores take bf16 X only with bf16
+//    weights, and one bf16 copy would be too coarse);
+//  * tc_kernel.  Work unit: 256 rows (eight consecutive 32-row groups, any
+//    block sizes) x one batch tile of N = 32..256 columns x one cluster
+//    rank's share of the columns of W, walked in stages of 32 columns:
+//      - a TMA warp copies the stage's rows of hi and lo for the batch tile
+//        straight into two MN-major B tiles (128-byte swizzle; rows and
+//        columns past the ends read as zeros);
+//      - sixteen producer warps, two per 32-row group taking alternate
+//        stages (one thread per row; all lanes of a warp share the group's
+//        block size and walk the blocks in lockstep), zero the row's 64 bytes
+//        of the stage and write the row's kept values that fall in it (bf16,
+//        exact) into two 128 x 32 A tiles (K-major, 64-byte swizzle); for
+//        m >= 16 at most three blocks meet a stage and are decoded in
+//        straight-line code;
+//      - an MMA warp issues, per stage and 128-row half, A*B_hi + A*B_lo for
+//        two K=16 steps into that half's TMEM accumulator (128 lanes x N fp32
+//        columns) and releases the stage with tcgen05.commit.
+//    At the end the ranks of a cluster add their partial accumulators: every
+//    rank writes its partial tile to workspace (L2-resident, coalesced),
+//    the cluster meets at one barrier, and each rank adds the partials of
+//    its slice of the rows in rank order (deterministic) and writes them to
+//    Y.  (Pushing the rows through distributed shared memory instead moved
+//    only ~10 bytes/clock per SM.)
+// Per stage the shared memory moves the MMA operands (96 KB at N = 256), the
+// copied B tiles and the A rows; with the split done beforehand that stays
+// near what the tensor cores need for the stage's multiplies.
 //
 // Numerics: weights are exact; |x - hi - lo| <= 2^-16 |x| (two round-to-
 // nearest bf16 steps), products are exact and accumulate in fp32, so
@@ -48,6 +54,7 @@
 #include <cooperative_groups.h>
 #include <cuda_bf16.h>
 
+#include <algorithm>
 #include <cstring>
 
 namespace darb {
@@ -58,36 +65,29 @@ namespace cg = cooperative_groups;
 constexpr int kRows = 256;                       // rows per CTA
 constexpr int kCtaGroups = kRows / kSlots;       // 32-row groups per CTA
 constexpr int kK = 32;                           // columns of W per stage
-constexpr int kProducerWarps = 8;                // kept values -> A, one thread per row
-constexpr int kConverterWarps = 12;              // staged activations -> B_hi, B_lo
-constexpr int kConverters = kConverterWarps * 32;
-constexpr int kTmaWarp = kProducerWarps + kConverterWarps;   // activation copies
+constexpr int kRowWarps = kRows / 32;            // warps that cover the CTA's rows once
+constexpr int kProducerWarps = 2 * kRowWarps;    // kept values -> A: two warps per group, alternate stages
+constexpr int kTmaWarp = kProducerWarps;         // activation copies
 constexpr int kMmaWarp = kTmaWarp + 1;           // TMEM owner, MMA issue
 constexpr int kThreads = (kMmaWarp + 1) * 32;
 constexpr int kARow = kK * 2;                    // bytes of one A row (bf16, 64-byte swizzle)
 constexpr int kAHalf = 128 * kARow;              // one 128-row A tile
-constexpr int kMaxStages = 6;
-constexpr int kMaxX = 3;
-constexpr int kXSlot = 32 * 1024;                // bytes of one staging slot
+constexpr int kBox = 64;                         // batch columns of one B box (128 bytes of bf16)
+constexpr int kMaxStages = 8;
 constexpr int kStageOff = 1024;                  // after the barriers; 1024-byte aligned
 constexpr size_t kSmemLimit = 227 * 1024;
 
-static_assert(kStageOff % 1024 == 0, "stages must start on a swizzle-atom boundary");
-
-// One bf16 B tile: 64-column x 8-row atoms of 1 KB, four K groups per 64 columns.
-__host__ __device__ constexpr int b_tile_bytes(int N) { return (N + 63) / 64 * 4096; }
+// One bf16 B tile: boxes of 64 columns x 32 rows (4 KB), i.e. 8-row x
+// 128-byte atoms, four K groups per 64 columns.
+__host__ __device__ constexpr int b_tile_bytes(int N) { return (N + kBox - 1) / kBox * 4096; }
 // An MMA stage: the two A halves, B_hi and B_lo.
 __host__ __device__ constexpr int mma_stage_bytes(int N) { return 2 * kAHalf + 2 * b_tile_bytes(N); }
-// Stages per staging slot: a slot holds 32 columns x 32R rows per 32-column box.
-__host__ __device__ constexpr int x_stages(int N) { return kXSlot / (N * kK * 4); }
 
 __host__ __device__ constexpr uint32_t tmem_cols(int N) { return 2 * N < 32 ? 32u : uint32_t(2 * N); }
 
 struct Plan {
     int N;          // batch tile width: 32, 64, 128 or 256
     int nstages;    // MMA stages in the ring
-    int nx;         // staging slots in the ring
-    int prows;      // rows of the partial-sum buffer per reduction round (256 or 128)
     size_t smem;    // dynamic shared memory, including 1024 bytes of alignment slack
 };
 
@@ -95,14 +95,9 @@ inline Plan plan_for(int N) {
     Plan p{};
     p.N = N;
     const size_t budget = kSmemLimit - 1024 - kStageOff;
-    // three staging slots when that leaves room for four MMA stages, else two
-    p.nx = size_t(4) * mma_stage_bytes(N) + size_t(kMaxX) * kXSlot <= budget ? kMaxX : 2;
-    p.nstages = static_cast<int>((budget - size_t(p.nx) * kXSlot) / mma_stage_bytes(N));
+    p.nstages = static_cast<int>(budget / mma_stage_bytes(N));
     if (p.nstages > kMaxStages) p.nstages = kMaxStages;
-    const size_t area = size_t(p.nstages) * mma_stage_bytes(N) + size_t(p.nx) * kXSlot;
-    // the partial-sum buffer holds ksplit * ceil(prows / ksplit) <= prows + 7 rows
-    p.prows = size_t(kRows + 8) * (N + 4) * 4 <= area ? kRows : 128;
-    p.smem = 1024 + kStageOff + area;
+    p.smem = 1024 + kStageOff + size_t(p.nstages) * mma_stage_bytes(N);
     return p;
 }
 
@@ -112,30 +107,56 @@ inline Plan plan_for(int N) {
 __device__ __forceinline__ int a_row(int r) { return (r >> 3) * 512 + (r & 7) * kARow; }
 __device__ __forceinline__ int a_swz(int r) { return ((r >> 1) & 3) << 4; }
 
-__device__ __forceinline__ uint32_t pack_hi_lo(float a, float b, uint32_t *lo) {
+// x -> (hi, lo) as bf16 bits: hi = bf16(x), lo = bf16(x - hi), both rounded to nearest.
+__device__ __forceinline__ void split2(float a, float b, uint32_t *hi, uint32_t *lo) {
     const __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
     const __nv_bfloat162 l = __floats2bfloat162_rn(a - __low2float(h), b - __high2float(h));
+    *hi = *reinterpret_cast<const uint32_t *>(&h);
     *lo = *reinterpret_cast<const uint32_t *>(&l);
-    return *reinterpret_cast<const uint32_t *>(&h);
+}
+
+// hi, lo: cols x batch bf16 with row pitch ldw (a multiple of 8).  Each thread
+// takes four consecutive batch columns of one row.
+__global__ void __launch_bounds__(256)
+split_kernel(const float *X, int64_t ldx, int64_t batch, int64_t cols, uint16_t *hi, uint16_t *lo, int64_t ldw) {
+    pdl_launch_dependents();
+    pdl_wait_previous();   // X may come from the previous kernel; the workspace may still be read by it
+    const int64_t q4 = (batch + 3) / 4;
+    const bool vec = (ldx & 3) == 0 && (reinterpret_cast<uintptr_t>(X) & 15) == 0;
+    for (int64_t i = int64_t(blockIdx.x) * blockDim.x + threadIdx.x; i < cols * q4;
+         i += int64_t(gridDim.x) * blockDim.x) {
+        const int64_t k = i / q4, b = (i - k * q4) * 4;
+        const float *x = X + k * ldx + b;
+        float4 v;
+        if (vec && b + 4 <= batch) {
+            v = __ldg(reinterpret_cast<const float4 *>(x));
+        } else {
+            v.x = __ldg(x);
+            v.y = b + 1 < batch ? __ldg(x + 1) : 0.0f;
+            v.z = b + 2 < batch ? __ldg(x + 2) : 0.0f;
+            v.w = b + 3 < batch ? __ldg(x + 3) : 0.0f;
+        }
+        uint2 h, l;
+        split2(v.x, v.y, &h.x, &l.x);
+        split2(v.z, v.w, &h.y, &l.y);
+        // ldw is a multiple of 8 and b of 4, so b + 4 <= ldw: 8-byte aligned, inside the row
+        *reinterpret_cast<uint2 *>(hi + k * ldw + b) = h;
+        *reinterpret_cast<uint2 *>(lo + k * ldw + b) = l;
+    }
 }
 
 __global__ void __launch_bounds__(kThreads, 1)
-tc_kernel(const __grid_constant__ CUtensorMap xmap, Format f, int ksplit, int nstages, int nx, int N, int prows,
-          int64_t batch, float *Y, int64_t ldy, int early) {
+tc_kernel(const __grid_constant__ CUtensorMap hmap, const __grid_constant__ CUtensorMap lmap, Format f, int ksplit,
+          int nstages, int N, int64_t batch, float *Y, int64_t ldy, float *part, int early) {
     extern __shared__ unsigned char sm_raw[];
     unsigned char *sm = reinterpret_cast<unsigned char *>((reinterpret_cast<uintptr_t>(sm_raw) + 1023) &
                                                           ~uintptr_t(1023));
-    uint64_t *full = reinterpret_cast<uint64_t *>(sm);     // MMA stage written (producers, converters)
+    uint64_t *full = reinterpret_cast<uint64_t *>(sm);     // MMA stage written (producers, TMA)
     uint64_t *empty = full + kMaxStages;                   // MMA stage consumed (commit)
-    uint64_t *xfull = empty + kMaxStages;                  // staging slot landed (TMA)
-    uint64_t *xempty = xfull + kMaxX;                      // staging slot converted (converters)
-    uint64_t *done = xempty + kMaxX;
+    uint64_t *done = empty + kMaxStages;
     uint32_t *s_tmem = reinterpret_cast<uint32_t *>(done + 1);
     unsigned char *const stages = sm + kStageOff;
     const int sbytes = mma_stage_bytes(N), bbytes = b_tile_bytes(N);
-    unsigned char *const xring = stages + size_t(nstages) * sbytes;
-    const int R = x_stages(N);                             // stages per staging slot
-    const int xbox = R * kK * 128;                         // bytes of one 32-column box of a slot
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int tile = blockIdx.x / ksplit, rank = blockIdx.x % ksplit;
@@ -148,12 +169,8 @@ tc_kernel(const __grid_constant__ CUtensorMap xmap, Format f, int ksplit, int ns
     pdl_launch_dependents();
     if (tid == 0) {
         for (int s = 0; s < kMaxStages; ++s) {
-            mbar_init(&full[s], kProducerWarps + kConverterWarps);
+            mbar_init(&full[s], kRowWarps + 1);   // the stage's producer warps and the TMA thread
             mbar_init(&empty[s], 1);
-        }
-        for (int x = 0; x < kMaxX; ++x) {
-            mbar_init(&xfull[x], 1);
-            mbar_init(&xempty[x], kConverterWarps);
         }
         mbar_init(done, 1);
         fence_mbar_init();
@@ -162,7 +179,10 @@ tc_kernel(const __grid_constant__ CUtensorMap xmap, Format f, int ksplit, int ns
         tmem_alloc(s_tmem, tcols);
         tmem_relinquish();
     }
-    if (warp == kTmaWarp && lane == 0) prefetch_tensormap(&xmap);
+    if (warp == kTmaWarp && lane == 0) {
+        prefetch_tensormap(&hmap);
+        prefetch_tensormap(&lmap);
+    }
     tc_fence_before_sync();
     __syncthreads();
     tc_fence_after_sync();
@@ -170,11 +190,12 @@ tc_kernel(const __grid_constant__ CUtensorMap xmap, Format f, int ksplit, int ns
     bool ok = true;
 
     if (warp < kProducerWarps) {
-        // ---- producers: thread t owns row t of the CTA (half t / 128 of the tile);
-        // warp w is group tile*8 + w, so m is uniform across the warp
+        // ---- producers: warp w covers group tile*8 + (w % 8), so m is uniform
+        // across it, on the stages of parity w / 8; thread t owns row t % 256
+        // of the CTA (half (t % 256) / 128 of the tile)
         if (!early) pdl_wait_previous();
-        const int t = tid, r = t & 127;
-        const int g = tile * kCtaGroups + warp;
+        const int t = tid & (kRows - 1), r = t & 127, par = warp / kRowWarps;
+        const int g = tile * kCtaGroups + (warp & (kRowWarps - 1));
         int m = 1, n = 0, nib = 1, nrows = 0;
         int64_t val_off = 0, off_off = 0;
         if (g < f.ngroups) {
@@ -196,11 +217,11 @@ tc_kernel(const __grid_constant__ CUtensorMap xmap, Format f, int ksplit, int ns
                 else o = __ldg(reinterpret_cast<const uint2 *>(f.offs + off_off) + rec);
             }
         };
-        // blocks of this rank's first stage start at jb = floor(k0 / m), rem = k0 - jb*m;
-        // each next stage moves k0 by 32 = q32*m + r32
-        const int k0first = ks0 * kK;
+        // blocks of this warp's first stage start at jb = floor(k0 / m), rem = k0 - jb*m;
+        // each next stage of the warp moves k0 by 64 = q64*m + r64
+        const int k0first = (ks0 + par) * kK;
         int jb = k0first / m, rem = k0first - jb * m;
-        const int q32 = kK / m, r32 = kK - q32 * m;
+        const int q64 = 2 * kK / m, r64 = 2 * kK - q64 * m;
         // chunk cc in (cv, co), cc+1 and cc+2 prefetched
         int cc = jb >> 3;
         uint4 cv = make_uint4(0, 0, 0, 0), v1 = cv, v2 = cv;
@@ -217,9 +238,9 @@ tc_kernel(const __grid_constant__ CUtensorMap xmap, Format f, int ksplit, int ns
         auto offset = [nib](const uint2 &o, int q) -> uint32_t {
             return nib ? (o.x >> (4 * q)) & 15u : ((q < 4 ? o.x : o.y) >> (8 * (q & 3))) & 255u;
         };
-        int s = 0;
-        uint32_t phase = 0;   // parity of the current use of stage s
-        for (int it = 0; it < nst; ++it) {
+        int s = par % nstages;
+        uint32_t phase = par >= nstages ? 1u : 0u;   // parity of the current use of stage s
+        for (int it = par; it < nst; it += 2) {
             if (it >= nstages && !__all_sync(0xFFFFFFFFu, mbar_wait(&empty[s], phase ^ 1u, false))) {
                 ok = false;   // the whole warp leaves together
                 break;
@@ -243,8 +264,8 @@ tc_kernel(const __grid_constant__ CUtensorMap xmap, Format f, int ksplit, int ns
             } else {
                 // blocks j with j*m < k0 + 32, from jb on: the same for every lane
                 for (int j = jb; j < n && j * m < k0 + kK; ++j) {
-                    if ((j >> 3) != cc) {   // step into the next chunk, prefetch two ahead
-                        cc = j >> 3;
+                    while ((j >> 3) != cc) {   // step through to j's chunk, prefetch two ahead
+                        ++cc;
                         cv = v1;
                         co = o1;
                         v1 = v2;
@@ -257,13 +278,13 @@ tc_kernel(const __grid_constant__ CUtensorMap xmap, Format f, int ksplit, int ns
                         *reinterpret_cast<uint16_t *>(row + ((2 * p) ^ swz)) = value(cv, q);
                 }
             }
-            jb += q32;
-            rem += r32;
+            jb += q64;
+            rem += r64;
             if (rem >= m) {
                 rem -= m;
                 ++jb;
             }
-            if (m >= 16 && (jb >> 3) != cc) {   // at most one chunk per stage when m >= 16
+            if (m >= 16 && (jb >> 3) != cc) {   // at most one chunk per step when m >= 16
                 cc = jb >> 3;
                 cv = v1;
                 co = o1;
@@ -274,80 +295,34 @@ tc_kernel(const __grid_constant__ CUtensorMap xmap, Format f, int ksplit, int ns
             fence_proxy_async_smem();   // the tensor core reads A through the async proxy
             __syncwarp();
             if (lane == 0) mbar_arrive(&full[s]);
-            if (++s == nstages) {
-                s = 0;
+            s += 2;
+            while (s >= nstages) {
+                s -= nstages;
                 phase ^= 1u;
-            }
-        }
-    } else if (warp < kTmaWarp) {
-        // ---- converters: staged fp32 (32-column boxes) -> B_hi, B_lo (64-column atoms)
-        const int ct = tid - kProducerWarps * 32;
-        const int units = N * (kK / 8);   // (row k of the stage, 8 batch columns)
-        int s = 0, x = 0, sub = 0;
-        uint32_t phase = 0, xphase = 0;
-        for (int it = 0; it < nst; ++it) {
-            if (it >= nstages && !__all_sync(0xFFFFFFFFu, mbar_wait(&empty[s], phase ^ 1u, false))) {
-                ok = false;
-                break;
-            }
-            if (!__all_sync(0xFFFFFFFFu, mbar_wait(&xfull[x], xphase, false))) {
-                ok = false;
-                break;
-            }
-            const unsigned char *xs = xring + size_t(x) * kXSlot + sub * (kK * 128);
-            unsigned char *bhi = stages + size_t(s) * sbytes + 2 * kAHalf, *blo = bhi + bbytes;
-            for (int u = ct; u < units; u += kConverters) {
-                const int k = u & (kK - 1), nc = u >> 5;   // lanes: consecutive rows k, conflict-free
-                const unsigned char *src = xs + (nc >> 2) * xbox + k * 128;
-                const int c4 = (nc & 3) * 2;
-                const float4 a4 = *reinterpret_cast<const float4 *>(src + ((c4 ^ (k & 7)) << 4));
-                const float4 b4 = *reinterpret_cast<const float4 *>(src + (((c4 + 1) ^ (k & 7)) << 4));
-                uint4 hv, lv;
-                hv.x = pack_hi_lo(a4.x, a4.y, &lv.x);
-                hv.y = pack_hi_lo(a4.z, a4.w, &lv.y);
-                hv.z = pack_hi_lo(b4.x, b4.y, &lv.z);
-                hv.w = pack_hi_lo(b4.z, b4.w, &lv.w);
-                const int off = (nc >> 3) * 4096 + (k >> 3) * 1024 + (k & 7) * 128 + (((nc & 7) ^ (k & 7)) << 4);
-                *reinterpret_cast<uint4 *>(bhi + off) = hv;
-                *reinterpret_cast<uint4 *>(blo + off) = lv;
-            }
-            fence_proxy_async_smem();   // the tensor core reads B through the async proxy
-            __syncwarp();
-            if (lane == 0) {
-                mbar_arrive(&full[s]);
-                if (sub == R - 1 || it == nst - 1) mbar_arrive(&xempty[x]);
-            }
-            if (++s == nstages) {
-                s = 0;
-                phase ^= 1u;
-            }
-            if (++sub == R) {
-                sub = 0;
-                if (++x == nx) {
-                    x = 0;
-                    xphase ^= 1u;
-                }
             }
         }
     } else if (warp == kTmaWarp) {
-        // ---- activation rows into the staging ring, R stages per slot
+        // ---- the stage's rows of hi and lo, straight into the B tiles
         if (lane == 0) {
-            pdl_wait_previous();   // X may come from the previous kernel
-            const int nslots = (nst + R - 1) / R;
-            int x = 0;
-            uint32_t xphase = 0;
-            for (int sl = 0; sl < nslots; ++sl) {
-                if (sl >= nx && !mbar_wait(&xempty[x], xphase ^ 1u, false)) {
+            pdl_wait_previous();   // the split is the previous kernel
+            const int nbox = (N + kBox - 1) / kBox;
+            int s = 0;
+            uint32_t phase = 0;
+            for (int it = 0; it < nst; ++it) {
+                if (it >= nstages && !mbar_wait(&empty[s], phase ^ 1u, false)) {
                     ok = false;
                     break;
                 }
-                unsigned char *xs = xring + size_t(x) * kXSlot;
-                mbar_arrive_expect_tx(&xfull[x], static_cast<uint32_t>(kXSlot));
-                for (int b = 0; b < N / 32; ++b)
-                    tensor2d_g2s(xs + b * xbox, &xmap, static_cast<int>(n0) + 32 * b, (ks0 + sl * R) * kK, &xfull[x]);
-                if (++x == nx) {
-                    x = 0;
-                    xphase ^= 1u;
+                unsigned char *bhi = stages + size_t(s) * sbytes + 2 * kAHalf, *blo = bhi + bbytes;
+                mbar_arrive_expect_tx(&full[s], static_cast<uint32_t>(2 * bbytes));
+                const int k0 = (ks0 + it) * kK;
+                for (int b = 0; b < nbox; ++b) {
+                    tensor2d_g2s(bhi + b * 4096, &hmap, static_cast<int>(n0) + kBox * b, k0, &full[s]);
+                    tensor2d_g2s(blo + b * 4096, &lmap, static_cast<int>(n0) + kBox * b, k0, &full[s]);
+                }
+                if (++s == nstages) {
+                    s = 0;
+                    phase ^= 1u;
                 }
             }
         }
@@ -394,103 +369,112 @@ tc_kernel(const __grid_constant__ CUtensorMap xmap, Format f, int ksplit, int ns
     }
 
     // ---- epilogue: accumulators -> Y (through a cluster reduction when split)
-    if (warp < kProducerWarps) {
+    if (warp < kRowWarps) {
         if (!__all_sync(0xFFFFFFFFu, mbar_wait(done, 0, false))) ok = false;
         tc_fence_after_sync();
     }
     pdl_wait_previous();   // Y may still be read by the previous kernel
     const bool vec = (ldy & 3) == 0 && (reinterpret_cast<uintptr_t>(Y) & 15) == 0;
     if (ksplit == 1) {
-        if (warp < kProducerWarps) {
+        if (warp < kRowWarps) {
+            // as for the partial tiles below: turn each 32 x 32 block around in
+            // shared memory so that 8 lanes write 32 consecutive columns of a row
             const int g = tile * kCtaGroups + warp;
-            const int64_t row = g < f.ngroups ? f.rowmap[g * kSlots + lane] : -1;
+            float *tb = reinterpret_cast<float *>(stages) + warp * (32 * 36);
+            const uint32_t tl = tmem + (uint32_t(32 * (warp & 3)) << 16) + uint32_t((warp >> 2) * N);
+            int64_t rows8[8];   // matrix rows of the block rows this lane writes
+#pragma unroll
+            for (int i = 0; i < 8; ++i) rows8[i] = g < f.ngroups ? f.rowmap[g * kSlots + 4 * i + (lane >> 3)] : -1;
+#pragma unroll 1
+            for (int cb = 0; cb < N / 32; ++cb) {   // 32 registers of accumulator at a time
+                uint32_t v[32];
+                tmem_ld32(tl + cb * 32, v);
+                tmem_ld_wait();
+#pragma unroll
+                for (int i = 0; i < 8; ++i)
+                    reinterpret_cast<uint4 *>(tb + lane * 36)[i] = make_uint4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+                __syncwarp();
+                const int64_t c0 = n0 + cb * 32 + 4 * (lane & 7);
+#pragma unroll
+                for (int i = 0; i < 8; ++i) {
+                    const int rr = 4 * i + (lane >> 3);
+                    const float4 a4 = reinterpret_cast<const float4 *>(tb + rr * 36)[lane & 7];
+                    if (rows8[i] >= 0 && c0 < batch) {
+                        float *y = Y + rows8[i] * ldy + c0;
+                        if (vec && c0 + 4 <= batch) {
+                            *reinterpret_cast<float4 *>(y) = a4;
+                        } else {
+                            const float f4[4] = {a4.x, a4.y, a4.z, a4.w};
+                            for (int q = 0; q < 4 && c0 + q < batch; ++q) y[q] = f4[q];
+                        }
+                    }
+                }
+                __syncwarp();
+            }
+        }
+    } else {
+        // partial tiles [tile of the grid][rank][256 rows][N] in workspace
+        float *const mine = part + ((size_t(blockIdx.y) * (gridDim.x / ksplit) + tile) * ksplit + rank) *
+                                       size_t(kRows) * N;
+        if (warp < kRowWarps) {
+            // a lane holds one row; turn each 32 x 32 block around in shared memory
+            // (rows padded to 36 floats: conflict-free) so that every store
+            // instruction writes four whole 128-byte row segments
+            float *tb = reinterpret_cast<float *>(stages) + warp * (32 * 36);   // the rings are free now
             const uint32_t tl = tmem + (uint32_t(32 * (warp & 3)) << 16) + uint32_t((warp >> 2) * N);
 #pragma unroll 1
             for (int cb = 0; cb < N / 32; ++cb) {   // 32 registers of accumulator at a time
                 uint32_t v[32];
                 tmem_ld32(tl + cb * 32, v);
                 tmem_ld_wait();
-                const int64_t c0 = n0 + cb * 32;
-                if (row >= 0 && c0 < batch) {
-                    float *y = Y + row * ldy + c0;
-                    const int64_t cnt = batch - c0;
-                    if (vec && cnt >= 32) {
 #pragma unroll
-                        for (int i = 0; i < 8; ++i)
-                            reinterpret_cast<float4 *>(y)[i] =
-                                make_float4(__uint_as_float(v[4 * i]), __uint_as_float(v[4 * i + 1]),
-                                            __uint_as_float(v[4 * i + 2]), __uint_as_float(v[4 * i + 3]));
-                    } else {
+                for (int i = 0; i < 8; ++i)
+                    reinterpret_cast<uint4 *>(tb + lane * 36)[i] = make_uint4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+                __syncwarp();
 #pragma unroll
-                        for (int i = 0; i < 32; ++i)
-                            if (i < cnt) y[i] = __uint_as_float(v[i]);
-                    }
+                for (int i = 0; i < 8; ++i) {
+                    const int rr = 4 * i + (lane >> 3), c4 = lane & 7;   // row of the block, float4 in the row
+                    __stcg(reinterpret_cast<float4 *>(mine + size_t(warp * 32 + rr) * N + cb * 32) + c4,
+                           reinterpret_cast<const float4 *>(tb + rr * 36)[c4]);
                 }
+                __syncwarp();
             }
         }
-    } else {
-        cg::cluster_group cluster = cg::this_cluster();
-        float *P = reinterpret_cast<float *>(stages);   // [source rank][owned row][pst]; free once all MMAs are done
-        const int pst = N + 4;                          // padded row stride: conflict-free stores
-        const int rounds = kRows / prows;
-        const int own = (prows + ksplit - 1) / ksplit;  // rows each rank owns per round
+        cg::this_cluster().sync();   // release/acquire: every rank's partial tile is visible
+        const float *first = mine - size_t(rank) * kRows * N;   // rank 0's tile
+        const int own = (kRows + ksplit - 1) / ksplit;       // rows each rank adds up
+        const int r0 = rank * own, r1 = min(kRows, r0 + own);
         const int nq = N / 4;
-        cluster.sync();   // every rank's MMAs are done: the stage rings may be overwritten
-        for (int round = 0; round < rounds; ++round) {
-            if (warp < kProducerWarps && (prows == kRows || (warp >> 2) == round)) {
-                const int prow = (prows == kRows ? warp * 32 : (warp & 3) * 32) + lane;   // row of the round
-                const int owner = prow / own;
-                const uint32_t dst = cluster_addr(smem_addr(P + (rank * own + (prow - owner * own)) * pst),
-                                                  static_cast<uint32_t>(owner));
-                const uint32_t tl = tmem + (uint32_t(32 * (warp & 3)) << 16) + uint32_t((warp >> 2) * N);
+        const size_t sstride = size_t(kRows) * N / 4;         // float4s between two ranks' tiles
 #pragma unroll 1
-                for (int cb = 0; cb < N / 32; ++cb) {   // 32 registers of accumulator at a time
-                    uint32_t v[32];
-                    tmem_ld32(tl + cb * 32, v);
-                    tmem_ld_wait();
+        for (int e = tid; e < (r1 - r0) * nq; e += kThreads) {
+            const int crow = r0 + e / nq, c4 = e % nq;
+            const float4 *src4 = reinterpret_cast<const float4 *>(first + size_t(crow) * N) + c4;
+            float4 v[8];   // every rank's partial in flight at once (ksplit <= 8), added in rank order
 #pragma unroll
-                    for (int i = 0; i < 8; ++i)
-                        st_cluster_v4(dst + (cb * 32 + 4 * i) * 4, v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+            for (int i = 0; i < 8; ++i)
+                if (i < ksplit) v[i] = __ldcg(src4 + i * sstride);
+            float4 acc = v[0];
+#pragma unroll
+            for (int i = 1; i < 8; ++i)
+                if (i < ksplit) {
+                    acc.x += v[i].x;
+                    acc.y += v[i].y;
+                    acc.z += v[i].z;
+                    acc.w += v[i].w;
+                }
+            const int g = tile * kCtaGroups + crow / kSlots;
+            const int64_t row = g < f.ngroups ? f.rowmap[g * kSlots + crow % kSlots] : -1;
+            const int64_t c0 = n0 + 4 * c4;
+            if (row >= 0 && c0 < batch) {
+                float *y = Y + row * ldy + c0;
+                if (vec && c0 + 4 <= batch) {
+                    *reinterpret_cast<float4 *>(y) = acc;
+                } else {
+                    const float a4[4] = {acc.x, acc.y, acc.z, acc.w};
+                    for (int i = 0; i < 4 && c0 + i < batch; ++i) y[i] = a4[i];
                 }
             }
-            cluster.sync();   // the partial rows have landed in their owners
-            const int r0 = rank * own, r1 = min(prows, r0 + own);
-#pragma unroll 1
-            for (int e = tid; e < (r1 - r0) * nq; e += kThreads) {
-                const int pr = e / nq, c4 = e % nq;
-                const float4 *src4 = reinterpret_cast<const float4 *>(P + pr * pst) + c4;
-                const int sstride = own * pst / 4;   // float4s between two sources' copies of the row
-                float4 acc = src4[0];
-#pragma unroll 1
-                for (int s0 = 1; s0 < ksplit; s0 += 4) {   // four loads in flight, added in rank order
-                    float4 v[4];
-#pragma unroll
-                    for (int i = 0; i < 4; ++i)
-                        if (s0 + i < ksplit) v[i] = src4[(s0 + i) * sstride];
-#pragma unroll
-                    for (int i = 0; i < 4; ++i)
-                        if (s0 + i < ksplit) {
-                            acc.x += v[i].x;
-                            acc.y += v[i].y;
-                            acc.z += v[i].z;
-                            acc.w += v[i].w;
-                        }
-                }
-                const int crow = (prows == kRows ? 0 : round * 128) + r0 + pr;   // row of the CTA
-                const int g = tile * kCtaGroups + crow / kSlots;
-                const int64_t row = g < f.ngroups ? f.rowmap[g * kSlots + crow % kSlots] : -1;
-                const int64_t c0 = n0 + 4 * c4;
-                if (row >= 0 && c0 < batch) {
-                    float *y = Y + row * ldy + c0;
-                    if (vec && c0 + 4 <= batch) {
-                        *reinterpret_cast<float4 *>(y) = acc;
-                    } else {
-                        const float a4[4] = {acc.x, acc.y, acc.z, acc.w};
-                        for (int i = 0; i < 4 && c0 + i < batch; ++i) y[i] = a4[i];
-                    }
-                }
-            }
-            cluster.sync();   // the owner has read its buffer before the next round refills it
         }
     }
 
@@ -503,18 +487,16 @@ tc_kernel(const __grid_constant__ CUtensorMap xmap, Format f, int ksplit, int ns
     }
 }
 
-// Tensor map over X (cols x batch fp32, row pitch ldx floats) with boxes of
-// 32 columns x 32R rows and 128-byte swizzle; false if X cannot be described
-// (alignment).
-inline bool make_xmap(CUtensorMap *map, const float *X, int64_t ldx, int64_t batch, int64_t cols, int N) {
-    if (X == nullptr || reinterpret_cast<uintptr_t>(X) % 16 != 0 || (ldx * 4) % 16 != 0) return false;
+// Tensor map over one bf16 part of X (cols x batch, row pitch ldw elements)
+// with 64-column x 32-row boxes and 128-byte swizzle.
+inline bool make_part_map(CUtensorMap *map, const uint16_t *part, int64_t ldw, int64_t batch, int64_t cols) {
     PFN_cuTensorMapEncodeTiled_v12000 enc = tensor_map_encoder();
     if (enc == nullptr) return false;
     const cuuint64_t dims[2] = {cuuint64_t(batch), cuuint64_t(cols)};
-    const cuuint64_t strides[1] = {cuuint64_t(ldx) * 4};
-    const cuuint32_t box[2] = {32, cuuint32_t(kK * x_stages(N))};
+    const cuuint64_t strides[1] = {cuuint64_t(ldw) * 2};
+    const cuuint32_t box[2] = {cuuint32_t(kBox), cuuint32_t(kK)};
     const cuuint32_t estr[2] = {1, 1};
-    return enc(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, const_cast<float *>(X), dims, strides, box, estr,
+    return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<uint16_t *>(part), dims, strides, box, estr,
                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
@@ -525,7 +507,7 @@ inline int tile_width(int64_t batch) {
     return N;
 }
 
-// Clusters of `ksplit` CTAs of this kernel that can be resident at once (0 if unknown).
+// Clusters of `ksplit` CTAs of this kernel that can be resident at once (-1 if unknown).
 inline int active_clusters(int ksplit, const Plan &p) {
     static int cache[4][9] = {};
     const int wi = p.N == 32 ? 0 : p.N == 64 ? 1 : p.N == 128 ? 2 : 3;
@@ -570,15 +552,14 @@ inline int pick_split(int64_t units, int KS, const Plan &p) {
     return best;
 }
 
-// cudaErrorNotSupported when the call does not fit this kernel (fp32 weights,
-// X not describable by a tensor map); the caller then takes the CUDA-core path.
+// cudaErrorNotSupported when the call does not fit this path (fp32 weights);
+// the caller then takes the CUDA-core path.  The split of X lives in
+// stream-ordered workspace from the device's default memory pool, taken and
+// returned on `stream` around the two kernels.
 inline cudaError_t launch(const Format &f, const float *X, int64_t ldx, int64_t batch, float *Y, int64_t ldy,
                           bool early, cudaStream_t stream) {
-    if (!f.bf16 || f.ngroups <= 0) return cudaErrorNotSupported;
-    CUtensorMap xmap;
-    std::memset(&xmap, 0, sizeof(xmap));
+    if (!f.bf16 || f.ngroups <= 0 || f.cols > (int64_t(1) << 31) - 1) return cudaErrorNotSupported;
     const Plan p = plan_for(tile_width(batch));
-    if (!make_xmap(&xmap, X, ldx, batch, f.cols, p.N)) return cudaErrorNotSupported;
     static const cudaError_t a = [] {
         size_t most = 0;
         for (int w = 32; w <= 256; w *= 2) most = plan_for(w).smem > most ? plan_for(w).smem : most;
@@ -589,9 +570,32 @@ inline cudaError_t launch(const Format &f, const float *X, int64_t ldx, int64_t 
     const int64_t NT = (batch + p.N - 1) / p.N;
     const int KS = static_cast<int>((f.cols + kK - 1) / kK);
     const int ksplit = pick_split(int64_t(T) * NT, KS, p);
-    const dim3 grid(static_cast<unsigned>(T * ksplit), static_cast<unsigned>(NT));
-    return launch_ex(tc_kernel, grid, dim3(kThreads), p.smem, stream, static_cast<unsigned>(ksplit), true, xmap, f,
-                     ksplit, p.nstages, p.nx, p.N, p.prows, batch, Y, ldy, early ? 1 : 0);
+    // workspace: hi and lo parts of X, then the partial tiles of a split
+    const int64_t ldw = (batch + 7) / 8 * 8;
+    const size_t part = (size_t(f.cols) * size_t(ldw) * 2 + 255) / 256 * 256;
+    const size_t partials = ksplit > 1 ? size_t(ksplit) * T * NT * kRows * p.N * 4 : 0;
+    void *ws = nullptr;
+    cudaError_t e = cudaMallocAsync(&ws, 2 * part + partials, stream);
+    if (e != cudaSuccess) return e;
+    uint16_t *hi = static_cast<uint16_t *>(ws), *lo = hi + part / 2;
+    float *pt = ksplit > 1 ? reinterpret_cast<float *>(static_cast<char *>(ws) + 2 * part) : nullptr;
+    CUtensorMap hmap, lmap;
+    std::memset(&hmap, 0, sizeof(hmap));
+    std::memset(&lmap, 0, sizeof(lmap));
+    if (!make_part_map(&hmap, hi, ldw, batch, f.cols) || !make_part_map(&lmap, lo, ldw, batch, f.cols)) {
+        cudaFreeAsync(ws, stream);
+        return cudaErrorNotSupported;
+    }
+    const int64_t items = f.cols * ((batch + 3) / 4);
+    const unsigned sgrid = static_cast<unsigned>(std::min<int64_t>((items + 255) / 256, int64_t(sm_count()) * 8));
+    e = launch_ex(split_kernel, dim3(sgrid), dim3(256), 0, stream, 1, true, X, ldx, batch, f.cols, hi, lo, ldw);
+    if (e == cudaSuccess) {
+        const dim3 grid(static_cast<unsigned>(T * ksplit), static_cast<unsigned>(NT));
+        e = launch_ex(tc_kernel, grid, dim3(kThreads), p.smem, stream, static_cast<unsigned>(ksplit), true, hmap,
+                      lmap, f, ksplit, p.nstages, p.N, batch, Y, ldy, pt, early ? 1 : 0);
+    }
+    const cudaError_t ef = cudaFreeAsync(ws, stream);
+    return e != cudaSuccess ? e : ef;
 }
 
 }  // namespace tc

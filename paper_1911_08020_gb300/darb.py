@@ -57,6 +57,7 @@ def lib():
                 "darb_sync_status": [P, S],
                 "darb_spmm": [P, P, I64, I64, P, I64, S],
                 "darb_spmm_ex": [P, P, I64, I64, P, I64, ctypes.c_int, S],
+                "darb_spmm_path": [P, I64, P, P],
                 "darb_lstm_step": [P, I64, I64, I64, P, P, P, P, P, P, S],
                 "darb_lstm_step_noalloc": [P, I64, I64, I64, P, P, P, P, P, P, S],
                 "darb_gru_step": [P, I64, I64, I64, P, P, P, P, P, S],
@@ -190,6 +191,13 @@ def darb_spmm_ex(h: Handle, X, Y=None, path: int = PATH_AUTO, stream=None):
         _check(lib().darb_spmm_ex(h.ptr, _ptr(X), ldx, batch, _ptr(Y), ldy, int(path), _stream(stream)),
                "darb_spmm_ex")
     return Y
+
+
+def darb_spmm_path(h: Handle, batch: int) -> tuple[int, int]:
+    """(path, kernels): the kernel family darb_spmm takes for this batch and its launches per call."""
+    path, kernels = ctypes.c_int(), ctypes.c_int32()
+    _check(lib().darb_spmm_path(h.ptr, int(batch), ctypes.byref(path), ctypes.byref(kernels)), "darb_spmm_path")
+    return path.value, kernels.value
 
 
 def darb_lstm_step(h: Handle, I: int, H: int, B: int, x, h_prev, c_prev, bias, h_out, c_out,

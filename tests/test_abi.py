@@ -109,6 +109,8 @@ def test_calls_reject_unknown_handles(L):
     assert L.darb_spmm(bogus, 4096, 1, 1, 8192, 1, None) == darb.ERR_INVALID_ARG
     for path in (darb.PATH_AUTO, darb.PATH_CUDA_CORES, darb.PATH_TENSOR_CORES, 3, -1):
         assert L.darb_spmm_ex(bogus, 4096, 1, 1, 8192, 1, path, None) == darb.ERR_INVALID_ARG
+    pth, nk = ctypes.c_int(), ctypes.c_int32()
+    assert L.darb_spmm_path(bogus, 256, ctypes.byref(pth), ctypes.byref(nk)) == darb.ERR_INVALID_ARG
     assert L.darb_lstm_step(bogus, 1, 1, 1, 4096, 4096, 4096, None, 8192, 8192, None) == darb.ERR_INVALID_ARG
     assert L.darb_gru_step(bogus, 1, 1, 1, 4096, 4096, None, None, 8192, None) == darb.ERR_INVALID_ARG
     assert L.darb_export(bogus, None, None, None, None) == darb.ERR_INVALID_ARG

@@ -1,6 +1,6 @@
 """The tensor-core product (densified tiles, tcgen05 kind::f16) against the oracle.
 
-darb_spmm sends bf16 weights with 128 or more batch columns to the tensor cores;
+darb_spmm sends bf16 weights with more than 32 batch columns to the tensor cores;
 darb_spmm_ex picks the path explicitly, so both kernel families are checked on
 the same inputs.  Activations enter the tensor cores as two bf16 parts
 (x = hi + lo, |x - hi - lo| <= 2^-16 |x|), so the error of that path is about
@@ -120,9 +120,9 @@ def test_tensor_path_strides_and_untouched_columns():
     stored, m = _case(g, rows, cols, (8, 32))
     h, ref = encode_both(stored, m, "bf16")
     try:
-        for B, pad in ((16, 4), (40, 8), (64, 0), (96, 12)):
+        for B, pad in ((16, 4), (40, 8), (64, 0), (96, 12), (33, 2), (130, 3)):
             Xbig = synth.activations(cols, B + pad, seed=B)
-            Xd = t(Xbig)[:, :B]                          # ldx = B + pad (a multiple of 4)
+            Xd = t(Xbig)[:, :B]                          # ldx = B + pad, any alignment
             Yd = torch.full((rows, B + 6), 7.0, device=dev())   # ldy = B + 6
             darb.darb_spmm_ex(h, Xd, Yd[:, :B], path=darb.PATH_TENSOR_CORES)
             Yr, A = oracle.darb_spmm(ref, Xbig[:, :B], with_absdot=True)
@@ -131,6 +131,23 @@ def test_tensor_path_strides_and_untouched_columns():
             assert np.all(Yh[:, B:] == 7.0), "wrote outside Y's columns"
     finally:
         darb.darb_destroy(h)
+
+
+def test_path_query_matches_the_automatic_choice():
+    g = np.random.default_rng(8)
+    w = (0.1 * g.standard_normal((64, 256))).astype(np.float32)
+    m = np.full(64, 16, np.int32)
+    h32, _ = encode_both(w, m, "f32")
+    h16, _ = encode_both(synth.f32_to_bf16_bits(w), m, "bf16")
+    try:
+        assert darb.darb_spmm_path(h32, 512) == (darb.PATH_CUDA_CORES, 1)
+        assert darb.darb_spmm_path(h16, 32) == (darb.PATH_CUDA_CORES, 1)
+        assert darb.darb_spmm_path(h16, 33) == (darb.PATH_TENSOR_CORES, 2)
+        with pytest.raises(darb.DarbError):
+            darb.darb_spmm_path(h16, 0)
+    finally:
+        darb.darb_destroy(h32)
+        darb.darb_destroy(h16)
 
 
 def test_tensor_path_refuses_what_it_cannot_take():
@@ -145,14 +162,10 @@ def test_tensor_path_refuses_what_it_cannot_take():
         with pytest.raises(darb.DarbError) as e:
             darb.darb_spmm_ex(h32, X, path=darb.PATH_TENSOR_CORES)
         assert e.value.status == darb.ERR_UNSUPPORTED
-        Xodd = t(synth.activations(128, 67, seed=2))[:, :66]   # ldx = 67: not a multiple of 4
-        with pytest.raises(darb.DarbError) as e:
-            darb.darb_spmm_ex(h16, Xodd, path=darb.PATH_TENSOR_CORES)
-        assert e.value.status == darb.ERR_UNSUPPORTED
-        # the automatic choice falls back to the CUDA cores for both
-        Y = darb.darb_spmm(h16, Xodd).cpu().numpy()
-        Yr, A = oracle.darb_spmm(ref16, Xodd.cpu().numpy(), with_absdot=True)
-        assert_product_close(Y, Yr, A, TOL["bf16"])
+        # the automatic choice falls back to the CUDA cores for fp32 weights
+        Y = darb.darb_spmm(h32, t(synth.activations(128, 200, seed=2))).cpu().numpy()
+        Yr, A = oracle.darb_spmm(ref32, synth.activations(128, 200, seed=2), with_absdot=True)
+        assert_product_close(Y, Yr, A, TOL["f32"])
         with pytest.raises(darb.DarbError) as e:
             darb.darb_spmm_ex(h16, X, path=7)
         assert e.value.status == darb.ERR_INVALID_ARG
