@@ -435,11 +435,43 @@ inline bool make_map(CUtensorMap *map, const float *A, int64_t ld, int64_t batch
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-// Grid shape: the largest row sets (most reuse of each staged activation row)
-// that still give two CTAs per SM with a cluster split of at most 8; then the
-// smallest cluster split that reaches about three CTAs per SM.
+// Grid shape of a plain product: row-set level l (sets of up to 2^l groups)
+// and cluster split k.
+// A CTA's work is proportional to 2^l / k and the launch takes
+// ceil(CTAs / resident CTAs) waves, so the cost is waves * 2^l / k; on a tie
+// the shape with fewer waves wins, then the larger sets (each staged
+// activation row serves more rows).  A partial second wave costs a whole one:
+// on FC6/FC7 at batch 16-32, sets of 4 groups split 8 ways (one wave) beat
+// sets of 2 groups split 8 ways (1.7 waves) by 25-35%.
 template <int LPR, int CPL>
-inline void grid_shape(const Format &f, int64_t tiles, int *level, unsigned *ksc) {
+inline void grid_shape(const Format &f, int64_t tiles, int per_sm, int *level, unsigned *ksc) {
+    const int64_t slots = int64_t(per_sm > 0 ? per_sm : 1) * sm_count();
+    double best = 1e300;
+    int64_t best_waves = 0;
+    *level = 0;
+    *ksc = 1;
+    for (int l = 3; l >= 0; --l) {
+        if ((1 << l) > max_set_groups<LPR, CPL>() || f.nsets[l] <= 0) continue;
+        for (unsigned k = 8; k >= 1; k /= 2) {
+            const int64_t ctas = int64_t(f.nsets[l]) * tiles * k;
+            const int64_t waves = (ctas + slots - 1) / slots;
+            const double cost = double(waves) * double(1 << l) / double(k);
+            if (cost < best * (1 - 1e-9) || (cost <= best * (1 + 1e-9) && waves < best_waves)) {
+                best = cost;
+                best_waves = waves;
+                *level = l;
+                *ksc = k;
+            }
+        }
+    }
+}
+
+// Grid shape of the fused RNN steps: each CTA also runs the cell epilogue
+// (arrival counters, the cell of the units it completes), so fewer, larger
+// CTAs win there: the largest row sets that still give two CTAs per SM with a
+// split of 8, then the smallest split that reaches three CTAs per SM.
+template <int LPR, int CPL>
+inline void grid_shape_rnn(const Format &f, int64_t tiles, int *level, unsigned *ksc) {
     const int64_t want_min = 2 * int64_t(sm_count()), target = 3 * int64_t(sm_count());
     *level = 0;
     for (int l = 3; l >= 0; --l) {
@@ -449,6 +481,21 @@ inline void grid_shape(const Format &f, int64_t tiles, int *level, unsigned *ksc
     }
     *ksc = 1;
     while (*ksc < 8 && int64_t(f.nsets[*level]) * tiles * *ksc < target) *ksc *= 2;
+}
+
+// CTAs of one batch_kernel instantiation resident per SM (shared memory is the limit).
+template <bool BF16, int LPR, int CPL, int MODE>
+inline int resident_per_sm() {
+    static const int n = [] {
+        int v = 0;
+        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&v, batch_kernel<BF16, LPR, CPL, MODE>, kThreads,
+                                                          smem_bytes<BF16>()) != cudaSuccess) {
+            cudaGetLastError();
+            v = 0;
+        }
+        return v > 0 ? v : 1;
+    }();
+    return n;
 }
 
 template <bool BF16, int LPR, int CPL, int MODE>
@@ -472,7 +519,8 @@ cudaError_t launch(const Format &f, const float *X, int64_t ldx, int64_t batch, 
     const int64_t tiles = (batch + kBt - 1) / kBt;
     int level;
     unsigned ksc;
-    grid_shape<LPR, CPL>(f, tiles, &level, &ksc);
+    if constexpr (MODE == kModeY) grid_shape<LPR, CPL>(f, tiles, resident_per_sm<BF16, LPR, CPL, MODE>(), &level, &ksc);
+    else grid_shape_rnn<LPR, CPL>(f, tiles, &level, &ksc);
     const dim3 grid(static_cast<unsigned>(f.nsets[level]) * ksc, static_cast<unsigned>(tiles));
     return launch_ex(batch_kernel<BF16, LPR, CPL, MODE>, grid, dim3(kThreads), smem, stream, ksc, true, f,
                      f.sets[level], X, ldx, batch, Y, ldy, xmap, hmap, ra, use_tma, early ? 1 : 0);
