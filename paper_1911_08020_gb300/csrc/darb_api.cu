@@ -27,6 +27,7 @@ struct darb_handle_s {
     std::vector<Group> groups;
     std::vector<int32_t> rowmap, rowloc, row_m;
     std::vector<darb::EncTile> enc_tiles;   // every encoder tile, resolved
+    int32_t max_tile = 0;                   // elements of the largest encoder tile (nb * m)
     std::vector<int2> sets;        // row sets of up to 1, 2, 4, 8 groups, concatenated
     int32_t nsets[4] = {0, 0, 0, 0};
     int64_t val_elems = 0, off_words = 0;
@@ -156,6 +157,7 @@ void build_layout(darb_handle_s *h, const int32_t *m) {
         }
     }
     h->enc_tiles.clear();
+    h->max_tile = 0;
     for (int64_t r = 0; r < rows; ++r) {
         const int32_t loc = h->rowloc[static_cast<size_t>(r)];
         const Group &g = h->groups[static_cast<size_t>(loc / kSlots)];
@@ -173,6 +175,7 @@ void build_layout(darb_handle_s *h, const int32_t *m) {
             t.val_base = g.val_off + rec * kChunk;
             t.off_base = g.off_off + rec * (g.nib ? 1 : 2);
             h->enc_tiles.push_back(t);
+            h->max_tile = std::max<int32_t>(h->max_tile, static_cast<int32_t>(nb * g.m));
         }
     }
 }
@@ -269,6 +272,7 @@ darb::EncodeTarget target_of(darb_handle_s *h) {
     darb::EncodeTarget t{};
     t.tiles = h->d_tiles;
     t.ntiles = static_cast<int32_t>(h->enc_tiles.size());
+    t.max_tile = h->max_tile;
     t.vals = h->d_vals;
     t.offs = h->d_offs;
     t.bf16 = h->wtype == DARB_BF16 ? 1 : 0;

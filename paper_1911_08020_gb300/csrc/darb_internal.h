@@ -80,6 +80,7 @@ struct __align__(16) EncTile {
 struct EncodeTarget {
     const EncTile *tiles;    // every encoder tile, row-major
     int32_t ntiles;
+    int32_t max_tile;        // elements of the largest tile, max over tiles of nb * m (zero padding included)
     void *vals;
     uint32_t *offs;
     int32_t bf16;

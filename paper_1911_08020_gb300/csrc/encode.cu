@@ -37,8 +37,14 @@ namespace {
 
 constexpr int kEncThreads = 256;
 
-template <bool BF16>
-__host__ __device__ constexpr int raw_bytes() { return kEncTileElems * (BF16 ? 2 : 4) + 128; }
+// Bytes of one stage: the largest tile of the handle plus room for its
+// 16-byte-misaligned start, in 128-byte units.  Sizing the ring to the
+// handle (not to the largest possible tile) lets short rows run with more
+// CTAs per SM, i.e. with more tiles in flight.
+inline int stage_bytes(const EncodeTarget &t) {
+    const int esz = t.bf16 ? 2 : 4;
+    return (t.max_tile * esz + 16 + 127) / 128 * 128;
+}
 
 template <bool BF16>
 __host__ __device__ constexpr int enc_stages() { return BF16 ? 3 : 2; }
@@ -46,8 +52,8 @@ __host__ __device__ constexpr int enc_stages() { return BF16 ? 3 : 2; }
 // shared memory: [0, 32) one mbarrier per stage, [32, 128) the descriptor of
 // the tile in each stage, then the stages' raw buffers
 template <bool BF16>
-__host__ __device__ constexpr size_t encode_smem() {
-    return 128 + size_t(enc_stages<BF16>()) * raw_bytes<BF16>();
+inline size_t encode_smem(int sbytes) {
+    return 128 + size_t(enc_stages<BF16>()) * sbytes;
 }
 static_assert(enc_stages<true>() * sizeof(EncTile) <= 96 && enc_stages<false>() * sizeof(EncTile) <= 96,
               "tile descriptors must fit in the shared-memory header");
@@ -84,14 +90,14 @@ __device__ __forceinline__ TileGeo tile_geo(const EncTile &d, const void *W, int
 
 template <bool BF16>
 __global__ void __launch_bounds__(kEncThreads)
-encode_kernel(EncodeTarget t, const void *W, int64_t ldw, int32_t *status) {
+encode_kernel(EncodeTarget t, const void *W, int64_t ldw, int32_t *status, int sbytes) {
     constexpr int kEsz = BF16 ? 2 : 4;
     constexpr int kStages = enc_stages<BF16>();
     using elem_t = typename std::conditional<BF16, uint16_t, uint32_t>::type;
     extern __shared__ __align__(128) unsigned char sm[];
     uint64_t *bar = reinterpret_cast<uint64_t *>(sm);        // one per stage
     EncTile *s_tile = reinterpret_cast<EncTile *>(sm + 32);   // the tile in each stage
-    unsigned char *const raw0 = sm + 128;                    // stage s at raw0 + s * raw_bytes
+    unsigned char *const raw0 = sm + 128;                    // stage s at raw0 + s * sbytes
     const int tid = threadIdx.x, lane = tid & 31;
 
     pdl_launch_dependents();
@@ -108,7 +114,7 @@ encode_kernel(EncodeTarget t, const void *W, int64_t ldw, int32_t *status) {
         const TileGeo g = tile_geo<BF16>(d, W, ldw);
         const uint32_t bytes = uint32_t(g.bhi - g.blo);
         mbar_arrive_expect_tx(&bar[s], bytes);
-        if (bytes > 0) bulk_g2s(raw0 + s * raw_bytes<BF16>() + g.blo, g.gaddr - g.off0 + g.blo, bytes, &bar[s]);
+        if (bytes > 0) bulk_g2s(raw0 + s * sbytes + g.blo, g.gaddr - g.off0 + g.blo, bytes, &bar[s]);
     };
 
     bool nan = false, ok = true;
@@ -138,10 +144,10 @@ encode_kernel(EncodeTarget t, const void *W, int64_t ldw, int32_t *status) {
         const TileGeo g = tile_geo<BF16>(d, W, ldw);
         const int m = d.m, nb = d.nb;
         const bool nib = m <= 16;
-        const int padded = nb * m;   // <= kEncTileElems
+        const int padded = nb * m;   // <= t.max_tile
         // element c of the tile sits at word c of `e`; fill the bytes the bulk
         // copy did not cover (unaligned head and tail) and zero the padding
-        elem_t *e = reinterpret_cast<elem_t *>(raw0 + s * raw_bytes<BF16>() + g.off0);
+        elem_t *e = reinterpret_cast<elem_t *>(raw0 + s * sbytes + g.off0);
         const int ehead = (g.blo - g.off0) / kEsz, etail = (g.bhi - g.off0) / kEsz;
         if (ehead > 0 || etail < padded) {   // the same for every thread
             const elem_t *src = reinterpret_cast<const elem_t *>(g.gaddr);
@@ -236,23 +242,37 @@ encode_kernel(EncodeTarget t, const void *W, int64_t ldw, int32_t *status) {
     if (__syncthreads_or(nan) && tid == 0) atomicOr(status, kStatusNaN);
 }
 
+// Largest dynamic shared memory any handle can ask for (tiles of kEncTileElems).
+template <bool BF16>
+inline size_t encode_smem_max() {
+    return encode_smem<BF16>((kEncTileElems * (BF16 ? 2 : 4) + 16 + 127) / 128 * 128);
+}
+
+template <bool BF16>
+cudaError_t launch_encode_t(const EncodeTarget &t, const void *W, int64_t ldw, int32_t *status,
+                            cudaStream_t stream) {
+    static const cudaError_t a = allow_smem(encode_kernel<BF16>, encode_smem_max<BF16>());
+    if (a != cudaSuccess) return a;
+    const int sbytes = stage_bytes(t);
+    const size_t smem = encode_smem<BF16>(sbytes);
+    // resident CTAs per SM at this handle's ring size (shared memory or threads bound it)
+    int per_sm = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, encode_kernel<BF16>, kEncThreads, smem) != cudaSuccess ||
+        per_sm <= 0) {
+        cudaGetLastError();
+        per_sm = 1;
+    }
+    const unsigned grid = static_cast<unsigned>(std::min<int64_t>(t.ntiles, per_sm * int64_t(sm_count())));
+    if (grid == 0) return cudaSuccess;
+    return launch_ex(encode_kernel<BF16>, dim3(grid), dim3(kEncThreads), smem, stream, 1, true, t, W, ldw, status,
+                     sbytes);
+}
+
 }  // namespace
 
 cudaError_t launch_encode(const EncodeTarget &t, const void *W, int64_t ldw, int32_t *status,
                           cudaStream_t stream) {
-    const int per_sm = t.bf16 ? 3 : 2;   // resident CTAs per SM at this kernel's shared memory
-    const unsigned grid = static_cast<unsigned>(std::min<int64_t>(t.ntiles, per_sm * int64_t(sm_count())));
-    if (grid == 0) return cudaSuccess;
-    if (t.bf16) {
-        static const cudaError_t a = allow_smem(encode_kernel<true>, encode_smem<true>());
-        if (a != cudaSuccess) return a;
-        return launch_ex(encode_kernel<true>, dim3(grid), dim3(kEncThreads), encode_smem<true>(), stream,
-                         1, true, t, W, ldw, status);
-    }
-    static const cudaError_t a = allow_smem(encode_kernel<false>, encode_smem<false>());
-    if (a != cudaSuccess) return a;
-    return launch_ex(encode_kernel<false>, dim3(grid), dim3(kEncThreads), encode_smem<false>(), stream,
-                     1, true, t, W, ldw, status);
+    return t.bf16 ? launch_encode_t<true>(t, W, ldw, status, stream) : launch_encode_t<false>(t, W, ldw, status, stream);
 }
 
 }  // namespace darb
