@@ -437,11 +437,12 @@ inline bool make_map(CUtensorMap *map, const float *A, int64_t ld, int64_t batch
 
 // Grid shape of a plain product: row-set level l (sets of up to 2^l groups)
 // and cluster split k.
-// A CTA's work is proportional to 2^l / k and the launch takes
-// ceil(CTAs / resident CTAs) waves, so the cost is waves * 2^l / k; on a tie
-// the shape with fewer waves wins, then the larger sets (each staged
-// activation row serves more rows).  A partial second wave costs a whole one:
-// on FC6/FC7 at batch 16-32, sets of 4 groups split 8 ways (one wave) beat
+// A CTA's work is proportional to 2^l / k plus a fixed cost (prologue,
+// reduction), about 0.2 in those units, and the launch takes
+// ceil(CTAs / resident CTAs) waves, so the cost is waves * (2^l / k + 0.2);
+// on a tie the shape with fewer waves wins, then the larger sets (each staged
+// activation row serves more rows).  Fitted to a sweep of every shape on
+// FC6/FC7 at batch 16-32, where sets of 4 groups split 8 ways (one wave) beat
 // sets of 2 groups split 8 ways (1.7 waves) by 25-35%.
 template <int LPR, int CPL>
 inline void grid_shape(const Format &f, int64_t tiles, int per_sm, int *level, unsigned *ksc) {
@@ -455,7 +456,7 @@ inline void grid_shape(const Format &f, int64_t tiles, int per_sm, int *level, u
         for (unsigned k = 8; k >= 1; k /= 2) {
             const int64_t ctas = int64_t(f.nsets[l]) * tiles * k;
             const int64_t waves = (ctas + slots - 1) / slots;
-            const double cost = double(waves) * double(1 << l) / double(k);
+            const double cost = double(waves) * (double(1 << l) / double(k) + 0.2);
             if (cost < best * (1 - 1e-9) || (cost <= best * (1 + 1e-9) && waves < best_waves)) {
                 best = cost;
                 best_waves = waves;

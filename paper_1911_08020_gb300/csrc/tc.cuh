@@ -64,29 +64,48 @@ namespace cg = cooperative_groups;
 
 constexpr int kRows = 256;                       // rows per CTA
 constexpr int kCtaGroups = kRows / kSlots;       // 32-row groups per CTA
-constexpr int kK = 32;                           // columns of W per stage
+// Columns of W per stage, KW: 32, or 64 for narrow batch tiles (N <= 64),
+// where the tensor cores finish a stage so fast that the per-stage hand-offs
+// would dominate.
 constexpr int kRowWarps = kRows / 32;            // warps that cover the CTA's rows once
 constexpr int kProducerWarps = 2 * kRowWarps;    // kept values -> A: two warps per group, alternate stages
 constexpr int kTmaWarp = kProducerWarps;         // activation copies
 constexpr int kMmaWarp = kTmaWarp + 1;           // TMEM owner, MMA issue
 constexpr int kThreads = (kMmaWarp + 1) * 32;
-constexpr int kARow = kK * 2;                    // bytes of one A row (bf16, 64-byte swizzle)
-constexpr int kAHalf = 128 * kARow;              // one 128-row A tile
 constexpr int kBox = 64;                         // batch columns of one B box (128 bytes of bf16)
 constexpr int kMaxStages = 8;
 constexpr int kStageOff = 1024;                  // after the barriers; 1024-byte aligned
 constexpr size_t kSmemLimit = 227 * 1024;
 
-// One bf16 B tile: boxes of 64 columns x 32 rows (4 KB), i.e. 8-row x
-// 128-byte atoms, four K groups per 64 columns.
-__host__ __device__ constexpr int b_tile_bytes(int N) { return (N + kBox - 1) / kBox * 4096; }
-// An MMA stage: the two A halves, B_hi and B_lo.
-__host__ __device__ constexpr int mma_stage_bytes(int N) { return 2 * kAHalf + 2 * b_tile_bytes(N); }
+// Layout of one stage width KW.  A rows are KW bf16 (64 or 128 bytes, with the
+// swizzle of that width: 8-row atoms of 512 or 1024 bytes); a B tile is made
+// of boxes of 64 batch columns x KW rows, i.e. KW/8 K groups of 8-row x
+// 128-byte atoms per 64 columns.
+template <int KW>
+struct Geo {
+    static constexpr int kARow = KW * 2;                     // bytes of one A row
+    static constexpr int kAHalf = 128 * kARow;               // one 128-row A tile
+    static constexpr int kAtom = 8 * kARow;                  // 8-row A atom
+    static constexpr uint32_t kALayout = KW == 32 ? kLayoutSw64 : kLayoutSw128;
+    static constexpr int kBCol = KW * 128;                   // one 64-column group of a B tile
+    static constexpr int kWindow = (KW - 1) / 16 + 2;        // blocks meeting a stage when m >= 16
+    static_assert(KW == 32 || KW == 64, "stage width");
+    // A row r (0..127) of a tile starts at row(r); kept value column p of it
+    // sits at row(r) + ((2p) ^ swz(r)): the swizzle XORs the 16-byte chunk bits
+    static __device__ __forceinline__ int row(int r) { return (r >> 3) * kAtom + (r & 7) * kARow; }
+    static __device__ __forceinline__ int swz(int r) { return KW == 32 ? ((r >> 1) & 3) << 4 : (r & 7) << 4; }
+    static __host__ __device__ constexpr int b_tile_bytes(int N) { return (N + kBox - 1) / kBox * kBCol; }
+    // an MMA stage: the two A halves, B_hi and B_lo
+    static __host__ __device__ constexpr int stage_bytes(int N) { return 2 * kAHalf + 2 * b_tile_bytes(N); }
+};
+
+__host__ __device__ constexpr int stage_width(int N) { return N <= 64 ? 64 : 32; }
 
 __host__ __device__ constexpr uint32_t tmem_cols(int N) { return 2 * N < 32 ? 32u : uint32_t(2 * N); }
 
 struct Plan {
     int N;          // batch tile width: 32, 64, 128 or 256
+    int KW;         // stage width
     int nstages;    // MMA stages in the ring
     size_t smem;    // dynamic shared memory, including 1024 bytes of alignment slack
 };
@@ -94,18 +113,14 @@ struct Plan {
 inline Plan plan_for(int N) {
     Plan p{};
     p.N = N;
+    p.KW = stage_width(N);
+    const int sb = p.KW == 64 ? Geo<64>::stage_bytes(N) : Geo<32>::stage_bytes(N);
     const size_t budget = kSmemLimit - 1024 - kStageOff;
-    p.nstages = static_cast<int>(budget / mma_stage_bytes(N));
+    p.nstages = static_cast<int>(budget / sb);
     if (p.nstages > kMaxStages) p.nstages = kMaxStages;
-    p.smem = 1024 + kStageOff + size_t(p.nstages) * mma_stage_bytes(N);
+    p.smem = 1024 + kStageOff + size_t(p.nstages) * sb;
     return p;
 }
-
-// An A tile row r (0..127) starts at a_row(r); kept value column p (0..31)
-// of it sits at a_row(r) + ((2p) ^ a_swz(r)): 2p is the byte offset, whose
-// 16-byte chunk bits the 64-byte swizzle XORs with (r / 2) % 4.
-__device__ __forceinline__ int a_row(int r) { return (r >> 3) * 512 + (r & 7) * kARow; }
-__device__ __forceinline__ int a_swz(int r) { return ((r >> 1) & 3) << 4; }
 
 // x -> (hi, lo) as bf16 bits: hi = bf16(x), lo = bf16(x - hi), both rounded to nearest.
 __device__ __forceinline__ void split2(float a, float b, uint32_t *hi, uint32_t *lo) {
@@ -145,9 +160,13 @@ split_kernel(const float *X, int64_t ldx, int64_t batch, int64_t cols, uint16_t 
     }
 }
 
+template <int KW>
 __global__ void __launch_bounds__(kThreads, 1)
 tc_kernel(const __grid_constant__ CUtensorMap hmap, const __grid_constant__ CUtensorMap lmap, Format f, int ksplit,
           int nstages, int N, int64_t batch, float *Y, int64_t ldy, float *part, int early) {
+    using G = Geo<KW>;
+    constexpr int kK = KW;
+    constexpr int kARow = G::kARow, kAHalf = G::kAHalf;
     extern __shared__ unsigned char sm_raw[];
     unsigned char *sm = reinterpret_cast<unsigned char *>((reinterpret_cast<uintptr_t>(sm_raw) + 1023) &
                                                           ~uintptr_t(1023));
@@ -156,7 +175,7 @@ tc_kernel(const __grid_constant__ CUtensorMap hmap, const __grid_constant__ CUte
     uint64_t *done = empty + kMaxStages;
     uint32_t *s_tmem = reinterpret_cast<uint32_t *>(done + 1);
     unsigned char *const stages = sm + kStageOff;
-    const int sbytes = mma_stage_bytes(N), bbytes = b_tile_bytes(N);
+    const int sbytes = G::stage_bytes(N), bbytes = G::b_tile_bytes(N);
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int tile = blockIdx.x / ksplit, rank = blockIdx.x % ksplit;
@@ -221,7 +240,7 @@ tc_kernel(const __grid_constant__ CUtensorMap hmap, const __grid_constant__ CUte
         // each next stage of the warp moves k0 by 64 = q64*m + r64
         const int k0first = (ks0 + par) * kK;
         int jb = k0first / m, rem = k0first - jb * m;
-        const int q64 = 2 * kK / m, r64 = 2 * kK - q64 * m;
+        const int q64 = 2 * kK / m, r64 = 2 * kK - q64 * m;   // two stages: 2*KW columns
         // chunk cc in (cv, co), cc+1 and cc+2 prefetched
         int cc = jb >> 3;
         uint4 cv = make_uint4(0, 0, 0, 0), v1 = cv, v2 = cv;
@@ -229,8 +248,8 @@ tc_kernel(const __grid_constant__ CUtensorMap hmap, const __grid_constant__ CUte
         load_chunk(cc, cv, co);
         load_chunk(cc + 1, v1, o1);
         load_chunk(cc + 2, v2, o2);
-        unsigned char *const row0 = stages + (t >> 7) * kAHalf + a_row(r);   // this row in stage 0
-        const int swz = a_swz(r);
+        unsigned char *const row0 = stages + (t >> 7) * kAHalf + G::row(r);   // this row in stage 0
+        const int swz = G::swz(r);
         auto value = [](const uint4 &v, int q) -> uint16_t {
             const uint32_t w = (q >> 1) == 0 ? v.x : (q >> 1) == 1 ? v.y : (q >> 1) == 2 ? v.z : v.w;
             return static_cast<uint16_t>((q & 1) ? w >> 16 : w);
@@ -251,9 +270,9 @@ tc_kernel(const __grid_constant__ CUtensorMap hmap, const __grid_constant__ CUte
                 reinterpret_cast<uint4 *>(row)[(c + lane) & (kARow / 16 - 1)] = make_uint4(0, 0, 0, 0);
             const int k0 = (ks0 + it) * kK;
             if (m >= 16) {
-                // blocks jb, jb+1, jb+2 (in chunk cc or cc+1) cover the stage
+                // blocks jb .. jb + kWindow - 1 (in chunk cc or cc+1) cover the stage
 #pragma unroll
-                for (int b = 0; b < 3; ++b) {
+                for (int b = 0; b < G::kWindow; ++b) {
                     const int j = jb + b;
                     const bool in1 = (j >> 3) != cc;
                     const int q = j & 7;
@@ -317,8 +336,8 @@ tc_kernel(const __grid_constant__ CUtensorMap hmap, const __grid_constant__ CUte
                 mbar_arrive_expect_tx(&full[s], static_cast<uint32_t>(2 * bbytes));
                 const int k0 = (ks0 + it) * kK;
                 for (int b = 0; b < nbox; ++b) {
-                    tensor2d_g2s(bhi + b * 4096, &hmap, static_cast<int>(n0) + kBox * b, k0, &full[s]);
-                    tensor2d_g2s(blo + b * 4096, &lmap, static_cast<int>(n0) + kBox * b, k0, &full[s]);
+                    tensor2d_g2s(bhi + b * G::kBCol, &hmap, static_cast<int>(n0) + kBox * b, k0, &full[s]);
+                    tensor2d_g2s(blo + b * G::kBCol, &lmap, static_cast<int>(n0) + kBox * b, k0, &full[s]);
                 }
                 if (++s == nstages) {
                     s = 0;
@@ -333,9 +352,9 @@ tc_kernel(const __grid_constant__ CUtensorMap hmap, const __grid_constant__ CUte
         const uint32_t sa0 = smem_addr(stages);
         // descriptors of stage 0; a stage is sbytes further on (the start
         // address field counts 16-byte units)
-        const uint64_t a0 = smem_desc(sa0, 16, 512, kLayoutSw64);
-        const uint64_t bh0 = smem_desc(sa0 + 2 * kAHalf, 4096, 1024, kLayoutSw128);
-        const uint64_t bl0 = smem_desc(sa0 + 2 * kAHalf + bbytes, 4096, 1024, kLayoutSw128);
+        const uint64_t a0 = smem_desc(sa0, 16, G::kAtom, G::kALayout);
+        const uint64_t bh0 = smem_desc(sa0 + 2 * kAHalf, G::kBCol, 1024, kLayoutSw128);
+        const uint64_t bl0 = smem_desc(sa0 + 2 * kAHalf + bbytes, G::kBCol, 1024, kLayoutSw128);
         int s = 0;
         uint32_t phase = 0;
         for (int it = 0; it < nst; ++it) {
@@ -488,13 +507,13 @@ tc_kernel(const __grid_constant__ CUtensorMap hmap, const __grid_constant__ CUte
 }
 
 // Tensor map over one bf16 part of X (cols x batch, row pitch ldw elements)
-// with 64-column x 32-row boxes and 128-byte swizzle.
-inline bool make_part_map(CUtensorMap *map, const uint16_t *part, int64_t ldw, int64_t batch, int64_t cols) {
+// with 64-column x kw-row boxes and 128-byte swizzle.
+inline bool make_part_map(CUtensorMap *map, const uint16_t *part, int64_t ldw, int64_t batch, int64_t cols, int kw) {
     PFN_cuTensorMapEncodeTiled_v12000 enc = tensor_map_encoder();
     if (enc == nullptr) return false;
     const cuuint64_t dims[2] = {cuuint64_t(batch), cuuint64_t(cols)};
     const cuuint64_t strides[1] = {cuuint64_t(ldw) * 2};
-    const cuuint32_t box[2] = {cuuint32_t(kBox), cuuint32_t(kK)};
+    const cuuint32_t box[2] = {cuuint32_t(kBox), cuuint32_t(kw)};
     const cuuint32_t estr[2] = {1, 1};
     return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<uint16_t *>(part), dims, strides, box, estr,
                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
@@ -508,6 +527,7 @@ inline int tile_width(int64_t batch) {
 }
 
 // Clusters of `ksplit` CTAs of this kernel that can be resident at once (-1 if unknown).
+template <int KW>
 inline int active_clusters(int ksplit, const Plan &p) {
     static int cache[4][9] = {};
     const int wi = p.N == 32 ? 0 : p.N == 64 ? 1 : p.N == 128 ? 2 : 3;
@@ -524,7 +544,7 @@ inline int active_clusters(int ksplit, const Plan &p) {
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     int n = 0;
-    if (cudaOccupancyMaxActiveClusters(&n, tc_kernel, &cfg) != cudaSuccess) {
+    if (cudaOccupancyMaxActiveClusters(&n, tc_kernel<KW>, &cfg) != cudaSuccess) {
         cudaGetLastError();
         n = 0;
     }
@@ -535,11 +555,12 @@ inline int active_clusters(int ksplit, const Plan &p) {
 
 // Cluster split: fewest waves per unit of work, i.e. the smallest
 // ceil(units / resident clusters) / ksplit, never more ranks than stages.
+template <int KW>
 inline int pick_split(int64_t units, int KS, const Plan &p) {
     int best = 1;
     double best_cost = 1e30;
     for (int s = 1; s <= 8 && s <= KS; ++s) {
-        int act = active_clusters(s, p);
+        int act = active_clusters<KW>(s, p);
         if (act <= 0) act = sm_count() / s;
         if (act <= 0) continue;
         const int64_t waves = (units + act - 1) / act;
@@ -552,24 +573,20 @@ inline int pick_split(int64_t units, int KS, const Plan &p) {
     return best;
 }
 
-// cudaErrorNotSupported when the call does not fit this path (fp32 weights);
-// the caller then takes the CUDA-core path.  The split of X lives in
-// stream-ordered workspace from the device's default memory pool, taken and
-// returned on `stream` around the two kernels.
-inline cudaError_t launch(const Format &f, const float *X, int64_t ldx, int64_t batch, float *Y, int64_t ldy,
-                          bool early, cudaStream_t stream) {
-    if (!f.bf16 || f.ngroups <= 0 || f.cols > (int64_t(1) << 31) - 1) return cudaErrorNotSupported;
-    const Plan p = plan_for(tile_width(batch));
+template <int KW>
+cudaError_t launch_kw(const Format &f, const float *X, int64_t ldx, int64_t batch, float *Y, int64_t ldy, bool early,
+                      const Plan &p, cudaStream_t stream) {
     static const cudaError_t a = [] {
         size_t most = 0;
-        for (int w = 32; w <= 256; w *= 2) most = plan_for(w).smem > most ? plan_for(w).smem : most;
-        return allow_smem(tc_kernel, most);
+        for (int w = 32; w <= 256; w *= 2)
+            if (stage_width(w) == KW) most = plan_for(w).smem > most ? plan_for(w).smem : most;
+        return allow_smem(tc_kernel<KW>, most);
     }();
     if (a != cudaSuccess) return a;
     const int T = (f.ngroups + kCtaGroups - 1) / kCtaGroups;
     const int64_t NT = (batch + p.N - 1) / p.N;
-    const int KS = static_cast<int>((f.cols + kK - 1) / kK);
-    const int ksplit = pick_split(int64_t(T) * NT, KS, p);
+    const int KS = static_cast<int>((f.cols + KW - 1) / KW);
+    const int ksplit = pick_split<KW>(int64_t(T) * NT, KS, p);
     // workspace: hi and lo parts of X, then the partial tiles of a split
     const int64_t ldw = (batch + 7) / 8 * 8;
     const size_t part = (size_t(f.cols) * size_t(ldw) * 2 + 255) / 256 * 256;
@@ -582,7 +599,7 @@ inline cudaError_t launch(const Format &f, const float *X, int64_t ldx, int64_t 
     CUtensorMap hmap, lmap;
     std::memset(&hmap, 0, sizeof(hmap));
     std::memset(&lmap, 0, sizeof(lmap));
-    if (!make_part_map(&hmap, hi, ldw, batch, f.cols) || !make_part_map(&lmap, lo, ldw, batch, f.cols)) {
+    if (!make_part_map(&hmap, hi, ldw, batch, f.cols, KW) || !make_part_map(&lmap, lo, ldw, batch, f.cols, KW)) {
         cudaFreeAsync(ws, stream);
         return cudaErrorNotSupported;
     }
@@ -591,11 +608,23 @@ inline cudaError_t launch(const Format &f, const float *X, int64_t ldx, int64_t 
     e = launch_ex(split_kernel, dim3(sgrid), dim3(256), 0, stream, 1, true, X, ldx, batch, f.cols, hi, lo, ldw);
     if (e == cudaSuccess) {
         const dim3 grid(static_cast<unsigned>(T * ksplit), static_cast<unsigned>(NT));
-        e = launch_ex(tc_kernel, grid, dim3(kThreads), p.smem, stream, static_cast<unsigned>(ksplit), true, hmap,
+        e = launch_ex(tc_kernel<KW>, grid, dim3(kThreads), p.smem, stream, static_cast<unsigned>(ksplit), true, hmap,
                       lmap, f, ksplit, p.nstages, p.N, batch, Y, ldy, pt, early ? 1 : 0);
     }
     const cudaError_t ef = cudaFreeAsync(ws, stream);
     return e != cudaSuccess ? e : ef;
+}
+
+// cudaErrorNotSupported when the call does not fit this path (fp32 weights);
+// the caller then takes the CUDA-core path.  The split of X lives in
+// stream-ordered workspace from the device's default memory pool, taken and
+// returned on `stream` around the two kernels.
+inline cudaError_t launch(const Format &f, const float *X, int64_t ldx, int64_t batch, float *Y, int64_t ldy,
+                          bool early, cudaStream_t stream) {
+    if (!f.bf16 || f.ngroups <= 0 || f.cols > (int64_t(1) << 31) - 1) return cudaErrorNotSupported;
+    const Plan p = plan_for(tile_width(batch));
+    return p.KW == 64 ? launch_kw<64>(f, X, ldx, batch, Y, ldy, early, p, stream)
+                      : launch_kw<32>(f, X, ldx, batch, Y, ldy, early, p, stream);
 }
 
 }  // namespace tc
