@@ -444,10 +444,40 @@ def run_gpu(args, world, rank, local):
     }
     if not args.no_rnn and not only:
         result["rnn"] = run_rnn(torch, darb, synth, peak)
+        result["assign"] = run_assign(torch, darb, wl, peak)
     if not args.no_e2e:
         result["e2e"] = run_e2e(args, wl, torch, darb)
     wl.close()
     return result
+
+
+def run_assign(torch, darb, wl, peak, reps=3):
+    """Block sizes from the weights (the step before encoding): a 4% top-K
+    magnitude mask of FC6 and FC7, timed with CUDA events around the call (it
+    synchronises).  Bytes: the radix passes and the counting pass each read W."""
+    out = {}
+    for mi, mat in enumerate(wl.mats):
+        W = mat["W"]
+        keep = mat["rows"] * mat["cols"] // 25
+        darb.darb_assign_from_weights(W, keep)          # warm-up
+        best = None
+        for _ in range(reps):
+            a = torch.cuda.Event(enable_timing=True)
+            b = torch.cuda.Event(enable_timing=True)
+            a.record()
+            darb.darb_assign_from_weights(W, keep)
+            b.record()
+            torch.cuda.synchronize()
+            ms = a.elapsed_time(b)
+            best = ms if best is None else min(best, ms)
+        passes = 3   # bf16: two radix passes and the count
+        nbytes = passes * mat["rows"] * mat["cols"] * 2
+        out["fc6" if mi == 0 else "fc7"] = {"keep_fraction": 0.04, "us": round(best * 1e3, 1),
+                                            "gbs": round(nbytes / (best * 1e-3) / 1e9, 1),
+                                            "hbm_frac": round(nbytes / (best * 1e-3) / 1e9 / peak, 4),
+                                            "note": "three reads of W (two radix passes and the row count)"
+                                                    " plus the host rounding rule and the copies"}
+    return out
 
 
 def run_rnn(torch, darb, synth, peak, reps=3):

@@ -80,6 +80,29 @@ DARB_API darb_status_t darb_assign_block_sizes(const int64_t *row_nnz, int64_t r
                                       int32_t m_min, int32_t m_max, int32_t *m_out);
 
 /*
+ * Block sizes from the weights themselves (Sec. 3.2): the K = `keep` weights
+ * of largest magnitude form the mask of irregular pruning (Sec. 2.2), used
+ * only to measure each row's density; darb_assign_block_sizes then turns the
+ * row counts into block sizes.  Weights tied with the K-th largest magnitude
+ * all count (the paper does not break such ties), so the counts may add up to
+ * slightly more than K.  Magnitudes are compared on the stored values (bf16
+ * or fp32); +0 and -0 tie; an infinity is the largest.
+ *   W        device, rows x cols row-major, leading dimension ldw (elements),
+ *            aligned to its element size
+ *   keep     1 <= keep <= rows * cols (and rows * cols < 2^32)
+ *   row_nnz_out  host int64[rows] receiving the counts, or NULL
+ *   m_out    host int32[rows] receiving the block sizes
+ * Runs on `stream` and synchronises it.  Device scratch (8 bytes per row) is
+ * kept by the library between calls, one buffer per device; concurrent calls
+ * take turns on it.
+ * Errors: DARB_ERR_INVALID_ARG; DARB_ERR_NONFINITE if W holds a NaN;
+ * DARB_ERR_UNSUPPORTED if rows * cols >= 2^32; DARB_ERR_OOM; DARB_ERR_CUDA.
+ */
+DARB_API darb_status_t darb_assign_from_weights(const void *W, darb_dtype_t wtype, int64_t rows, int64_t cols,
+                                                int64_t ldw, int64_t keep, int32_t m_min, int32_t m_max,
+                                                int64_t *row_nnz_out, int32_t *m_out, cudaStream_t stream);
+
+/*
  * BMWM encode (Sec. 3.1 steps (1)-(3), with the per-row block size of Sec. 3.2).
  *   W      device, rows x cols, row-major, leading dimension ldw >= cols
  *          (elements); fp32 or bf16 as wtype says.  Any alignment.

@@ -66,6 +66,8 @@ def load_library(path: str):
     lib.oracle_set_threads.argtypes = [ctypes.c_int]
     lib.oracle_set_threads.restype = ctypes.c_int
     lib.oracle_assign_block_sizes.argtypes = [P, I64, I64, I32, I32, P]
+    lib.oracle_topk_row_nnz_f32.argtypes = [P, I64, I64, I64, I64, P]
+    lib.oracle_topk_row_nnz_bf16.argtypes = [P, I64, I64, I64, I64, P]
     lib.oracle_block_pointers.argtypes = [P, I64, I64, P]
     lib.oracle_encode_f32.argtypes = [P, I64, I64, I64, P, P, P, P]
     lib.oracle_encode_bf16.argtypes = [P, I64, I64, I64, P, P, P, P]
@@ -73,7 +75,8 @@ def load_library(path: str):
     lib.oracle_darb_spmm.argtypes = [P, P, P, P, I64, I64, P, I64, I64, P, I64, P]
     lib.oracle_lstm_step.argtypes = [P, P, P, P, I64, I64, I64, P, P, P, P, P, P, P]
     lib.oracle_gru_step.argtypes = [P, P, P, P, I64, I64, I64, P, P, P, P, P, P]
-    for f in ("oracle_assign_block_sizes", "oracle_block_pointers", "oracle_encode_f32",
+    for f in ("oracle_assign_block_sizes", "oracle_topk_row_nnz_f32", "oracle_topk_row_nnz_bf16",
+              "oracle_block_pointers", "oracle_encode_f32",
               "oracle_encode_bf16", "oracle_masked_dense", "oracle_darb_spmm",
               "oracle_lstm_step", "oracle_gru_step"):
         getattr(lib, f).restype = ctypes.c_int
@@ -118,6 +121,19 @@ class Encoding:
         if self.dtype == "bf16":
             return (self.val.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
         return self.val.astype(np.float64)
+
+
+def topk_row_nnz(W: np.ndarray, keep: int, dtype: str | None = None) -> np.ndarray:
+    """Per-row count of the `keep` weights of largest magnitude (ties at the
+    threshold all count): the row densities of Sec. 3.2's first step."""
+    if dtype is None:
+        dtype = "bf16" if W.dtype == np.uint16 else "f32"
+    W = np.ascontiguousarray(W, dtype=np.uint16 if dtype == "bf16" else np.float32)
+    rows, cols = W.shape
+    out = np.zeros(rows, dtype=np.int64)
+    fn = _load().oracle_topk_row_nnz_bf16 if dtype == "bf16" else _load().oracle_topk_row_nnz_f32
+    _check(fn(_p(W), rows, cols, cols, int(keep), _p(out)), "topk_row_nnz")
+    return out
 
 
 def assign_block_sizes(row_nnz, cols: int, m_min: int = 1, m_max: int = 256) -> np.ndarray:

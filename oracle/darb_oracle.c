@@ -8,6 +8,9 @@
  * Every function is the plain definition of one step of the method, written as
  * loops in the paper's order, accumulating in double precision:
  *
+ *   oracle_topk_row_nnz_*      Sec. 3.2's first step with Sec. 2.2's irregular
+ *                              pruning: each row's count of the K weights of
+ *                              largest magnitude (the row density)
  *   oracle_assign_block_sizes  Sec. 3.2 (density-adaptive rounding rule)
  *   oracle_block_pointers      Sec. 3.1 step (1): ceil(cols / m) blocks per row
  *   oracle_encode_f32/_bf16    Sec. 3.1 BMWM steps (1)-(3), per-row block size
@@ -42,6 +45,58 @@ int oracle_set_threads(int n) {
     (void)n;
     return 1;
 #endif
+}
+
+/* ------------------------------------------------------------------------ */
+/* Sec. 3.2 starts from the mask of irregular pruning (Sec. 2.2: keep the K
+ * weights of largest magnitude) and only counts it: row r's density is its
+ * number of kept weights over cols.  Here: sort all magnitudes (widened
+ * exactly to double) in decreasing order, take the K-th one as the threshold t,
+ * and count per row the weights with |w| >= t.
+ * Reading: the paper does not say which of several weights equal to the K-th
+ * magnitude are kept; all of them count, so the counts may add up to more than
+ * K.  A NaN weight is rejected.                                               */
+static int cmp_desc(const void *a, const void *b) {
+    const double x = *(const double *)a, y = *(const double *)b;
+    return (x < y) - (x > y);
+}
+
+#define TOPK_BODY(LOAD)                                                               \
+    if (!W || !row_nnz || rows <= 0 || cols <= 0 || ldw < cols || keep < 1 ||         \
+        keep > rows * cols)                                                           \
+        return OR_INVALID;                                                            \
+    double *mag = (double *)malloc((size_t)(rows * cols) * sizeof(double));           \
+    if (!mag) return OR_INVALID;                                                      \
+    for (int64_t r = 0; r < rows; ++r)                                                \
+        for (int64_t c = 0; c < cols; ++c) {                                          \
+            const double v = LOAD(W[r * ldw + c]);                                    \
+            if (isnan(v)) {                                                           \
+                free(mag);                                                            \
+                return OR_NONFINITE;                                                  \
+            }                                                                         \
+            mag[r * cols + c] = fabs(v);                                              \
+        }                                                                             \
+    qsort(mag, (size_t)(rows * cols), sizeof(double), cmp_desc);                      \
+    const double t = mag[keep - 1];                                                   \
+    free(mag);                                                                        \
+    for (int64_t r = 0; r < rows; ++r) {                                              \
+        int64_t n = 0;                                                                \
+        for (int64_t c = 0; c < cols; ++c)                                            \
+            if (fabs(LOAD(W[r * ldw + c])) >= t) ++n;                                 \
+        row_nnz[r] = n;                                                               \
+    }                                                                                 \
+    return OR_OK;
+
+static double bf16_bits_value(uint16_t bits);
+
+int oracle_topk_row_nnz_f32(const float *W, int64_t rows, int64_t cols, int64_t ldw, int64_t keep,
+                            int64_t *row_nnz) {
+    TOPK_BODY((double))
+}
+
+int oracle_topk_row_nnz_bf16(const uint16_t *W, int64_t rows, int64_t cols, int64_t ldw, int64_t keep,
+                             int64_t *row_nnz) {
+    TOPK_BODY(bf16_bits_value)
 }
 
 /* ------------------------------------------------------------------------ */
@@ -102,6 +157,8 @@ static double bf16_value(uint16_t bits) {
     memcpy(&f, &u, sizeof f);
     return (double)f;
 }
+
+static double bf16_bits_value(uint16_t bits) { return bf16_value(bits); }
 
 static double f32_value(float f) { return (double)f; }
 

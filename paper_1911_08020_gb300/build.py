@@ -18,7 +18,7 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libdarb.so")
-SOURCES = ["darb_api.cu", "encode.cu", "spmm.cu", "spmm_batch.cu", "spmm_tc.cu", "rnn.cu", "rnn_batch.cu",
+SOURCES = ["darb_api.cu", "assign.cu", "encode.cu", "spmm.cu", "spmm_batch.cu", "spmm_tc.cu", "rnn.cu", "rnn_batch.cu",
            "noalloc.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 

@@ -7,6 +7,7 @@
 #include <algorithm>
 #include <cstdlib>
 #include <cstring>
+#include <map>
 #include <mutex>
 #include <new>
 #include <numeric>
@@ -505,6 +506,63 @@ darb_status_t darb_spmm_ex(darb_handle_t h, const float *X, int64_t ldx, int64_t
         return DARB_ERR_OOM;
     }
     return cuda_status(e);
+}
+
+darb_status_t darb_assign_from_weights(const void *W, darb_dtype_t wtype, int64_t rows, int64_t cols, int64_t ldw,
+                                       int64_t keep, int32_t m_min, int32_t m_max, int64_t *row_nnz_out,
+                                       int32_t *m_out, cudaStream_t stream) {
+    if (W == nullptr || m_out == nullptr || !valid_dtype(wtype)) return DARB_ERR_INVALID_ARG;
+    if (rows <= 0 || cols <= 0 || rows > kMaxDim || cols > kMaxDim || ldw < cols) return DARB_ERR_INVALID_ARG;
+    if (m_min < 1 || m_max < m_min || m_max > DARB_MAX_BLOCK) return DARB_ERR_INVALID_ARG;
+    const size_t esz = wtype == DARB_BF16 ? 2 : 4;
+    if (reinterpret_cast<uintptr_t>(W) % esz != 0) return DARB_ERR_INVALID_ARG;
+    if (keep < 1 || keep > rows * cols) return DARB_ERR_INVALID_ARG;
+    if (rows * cols >= (int64_t(1) << 32)) return DARB_ERR_UNSUPPORTED;
+    std::vector<int64_t> nnz;
+    try {
+        nnz.resize(static_cast<size_t>(rows));
+    } catch (const std::bad_alloc &) {
+        return DARB_ERR_OOM;
+    }
+    // scratch: selection state and histograms (4608 B), the NaN flag, the row counts
+    const size_t o_flag = 4608, o_rows = 4864;
+    // the call synchronises, so one scratch buffer per device serves every call
+    // (kept between calls, grown when a matrix has more rows; calls serialise on it)
+    static std::mutex scratch_mu;
+    static std::map<int, std::pair<void *, size_t>> scratch;
+    std::lock_guard<std::mutex> lk(scratch_mu);
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) {   // no device: the allocation below reports it
+        cudaGetLastError();
+        dev = -1;
+    }
+    auto &slot = scratch[dev];
+    const size_t need = o_rows + static_cast<size_t>(rows) * 8;
+    if (slot.second < need) {
+        if (slot.first) {
+            cudaDeviceSynchronize();
+            cudaFree(slot.first);
+            slot = {nullptr, 0};
+        }
+        void *p = nullptr;
+        const darb_status_t st = dev_alloc(&p, need);
+        if (st != DARB_OK) return st;
+        slot = {p, need};
+    }
+    void *work = slot.first;
+    char *b = static_cast<char *>(work);
+    int32_t nan_flag = 0;
+    cudaError_t e = darb::launch_topk_row_nnz(W, wtype == DARB_BF16, rows, cols, ldw, keep,
+                                              reinterpret_cast<int64_t *>(b + o_rows), work,
+                                              reinterpret_cast<int32_t *>(b + o_flag), stream);
+    if (e == cudaSuccess)
+        e = cudaMemcpyAsync(nnz.data(), b + o_rows, static_cast<size_t>(rows) * 8, cudaMemcpyDeviceToHost, stream);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(&nan_flag, b + o_flag, 4, cudaMemcpyDeviceToHost, stream);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(stream);
+    if (e != cudaSuccess) return DARB_ERR_CUDA;
+    if (nan_flag) return DARB_ERR_NONFINITE;
+    if (row_nnz_out) std::copy(nnz.begin(), nnz.end(), row_nnz_out);
+    return darb_assign_block_sizes(nnz.data(), rows, cols, m_min, m_max, m_out);
 }
 
 darb_status_t darb_spmm_path(darb_handle_t h, int64_t batch, darb_path_t *path, int32_t *kernels) {

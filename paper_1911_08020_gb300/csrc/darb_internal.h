@@ -139,6 +139,12 @@ int rnn_batch_tile(int64_t B);
 // Streaming multiprocessors of the current device (cached).
 int sm_count();
 
+// Row densities of Sec. 3.2's first step (assign.cu): row_nnz[r] = number of
+// weights of row r whose magnitude is >= the keep-th largest magnitude of W.
+// work: 4608 bytes of device scratch; nan_flag: device int, set if W has a NaN.
+cudaError_t launch_topk_row_nnz(const void *W, bool bf16, int64_t rows, int64_t cols, int64_t ldw, int64_t keep,
+                                int64_t *row_nnz, void *work, int32_t *nan_flag, cudaStream_t stream);
+
 // The argument checks of darb_lstm_step and the handle's read-only view, for
 // an entry point that brings its own scratch.  Allocates nothing.
 darb_status_t lstm_step_view(darb_handle_t h, int64_t I, int64_t H, int64_t B, const float *x,

@@ -52,6 +52,7 @@ def lib():
             P, I64, I32, S = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int32, ctypes.c_void_p
             sig = {
                 "darb_assign_block_sizes": [P, I64, I64, I32, I32, P],
+                "darb_assign_from_weights": [P, ctypes.c_int, I64, I64, I64, I64, I32, I32, P, P, S],
                 "darb_encode": [P, ctypes.c_int, I64, I64, I64, P, P, S],
                 "darb_reencode": [P, P, I64, S],
                 "darb_sync_status": [P, S],
@@ -139,6 +140,23 @@ def darb_assign_block_sizes(row_nnz, cols: int, m_min: int = 1, m_max: int = MAX
     _check(lib().darb_assign_block_sizes(nnz.ctypes.data, nnz.shape[0], int(cols), int(m_min),
                                          int(m_max), out.ctypes.data), "darb_assign_block_sizes")
     return out
+
+
+def darb_assign_from_weights(W, keep: int, m_min: int = 1, m_max: int = MAX_BLOCK, stream=None,
+                             ldw: int | None = None):
+    """(row_nnz, m): each row's count of the `keep` weights of largest magnitude of
+    the CUDA tensor W (rows x cols, float32 or bfloat16) and the block sizes they give."""
+    code = _dtype_code(W)
+    if W.dim() != 2 or not W.is_cuda or W.stride(1) != 1:
+        raise DarbError(ERR_INVALID_ARG, "darb_assign_from_weights: W must be a 2-D CUDA tensor with unit column stride")
+    rows, cols = W.shape
+    ldw = W.stride(0) if ldw is None else ldw
+    nnz = np.zeros(rows, dtype=np.int64)
+    m = np.zeros(rows, dtype=np.int32)
+    _check(lib().darb_assign_from_weights(_ptr(W), code, rows, cols, int(ldw), int(keep), int(m_min), int(m_max),
+                                          nnz.ctypes.data, m.ctypes.data, _stream(stream)),
+           "darb_assign_from_weights")
+    return nnz, m
 
 
 def darb_encode(W, m, stream=None, ldw: int | None = None) -> Handle:

@@ -34,6 +34,77 @@ def _kv(line):
     return dict(tok.split("=", 1) for tok in line.split())
 
 
+# --------------------------------------------------------------------------- top-K row densities
+def check_topk_worked_example(orc):
+    """Sec. 3.2 example through the mask: K = 28 of 4 x 32 weights, kept 12/6/5/5 -> m = 2/8/8/8."""
+    lines = _golden_lines("topk_worked_example.txt")
+    head = _kv(lines[0])
+    rows, cols, keep = int(head["rows"]), int(head["cols"]), int(head["keep"])
+    cases = [_kv(ln) for ln in lines[1:]]
+    g = np.random.default_rng(40)
+    for dtype in ("f32", "bf16"):
+        # row i: its first kept[i] columns hold large weights (magnitudes 1..2, distinct,
+        # random signs), the rest small ones (magnitude below 0.5)
+        W = (g.uniform(0.01, 0.5, (rows, cols)) * g.choice([-1, 1], (rows, cols))).astype(np.float32)
+        for c in cases:
+            r, k = int(c["row"]), int(c["kept"])
+            W[r, :k] = (1.0 + np.arange(k) / 64.0 + r / 8.0) * g.choice([-1, 1], k)
+        stored = W
+        if dtype == "bf16":
+            stored = (W.view(np.uint32) >> 16).astype(np.uint16)   # magnitudes chosen exact in bf16 above 1
+        nnz = orc.topk_row_nnz(stored, keep, dtype)
+        assert list(nnz) == [int(c["kept"]) for c in cases], (dtype, nnz)
+        m = orc.assign_block_sizes(nnz, cols)
+        assert list(m) == [int(c["block_size"]) for c in cases], (dtype, m)
+
+
+def _threshold_by_enumeration(mag, keep):
+    """The K-th largest magnitude as the unique candidate t with
+    #(|w| > t) < keep <= #(|w| >= t) (every distinct magnitude is tried)."""
+    for t in np.unique(mag):
+        if np.count_nonzero(mag > t) < keep <= np.count_nonzero(mag >= t):
+            return t
+    raise AssertionError("no threshold")
+
+
+def check_topk_random(orc):
+    """Brute force on small matrices: counts of |w| >= t with t found by enumeration;
+    with distinct magnitudes the counts add up to exactly K; K = all keeps every weight."""
+    g = np.random.default_rng(41)
+    for rows, cols in ((3, 4), (5, 7), (8, 33)):
+        n = rows * cols
+        # distinct magnitudes: a permutation of 1..n, random signs
+        W = (g.permutation(n).reshape(rows, cols) + 1).astype(np.float32) * g.choice([-1, 1], (rows, cols))
+        for keep in (1, 2, n // 3, n - 1, n):
+            nnz = orc.topk_row_nnz(W, keep, "f32")
+            t = _threshold_by_enumeration(np.abs(W), keep)
+            assert list(nnz) == list(np.count_nonzero(np.abs(W) >= t, axis=1)), (rows, cols, keep)
+            assert int(nnz.sum()) == keep
+        assert list(orc.topk_row_nnz(W, n, "f32")) == [cols] * rows
+        # K = 1 keeps only the largest magnitude's row
+        one = orc.topk_row_nnz(W, 1, "f32")
+        assert int(one.sum()) == 1 and one[np.unravel_index(np.argmax(np.abs(W)), W.shape)[0]] == 1
+
+
+def check_topk_ties(orc):
+    """Ties at the K-th magnitude all count; +0 and -0 tie; infinities are largest; NaN is refused."""
+    W = np.array([[2.0, -2.0, 1.0, 0.0], [-0.0, 2.0, -1.0, 3.0]], np.float32)
+    assert list(orc.topk_row_nnz(W, 1, "f32")) == [0, 1]          # 3
+    assert list(orc.topk_row_nnz(W, 2, "f32")) == [2, 2]          # 3, then three 2s tie
+    assert list(orc.topk_row_nnz(W, 5, "f32")) == [3, 3]          # the two 1s tie
+    assert list(orc.topk_row_nnz(W, 7, "f32")) == [4, 4]          # +0 and -0 tie
+    W2 = W.copy()
+    W2[0, 2] = -np.inf
+    assert list(orc.topk_row_nnz(W2, 1, "f32")) == [1, 0]
+    W2[1, 1] = np.nan
+    try:
+        orc.topk_row_nnz(W2, 1, "f32")
+    except orc.OracleError as e:
+        assert e.status == 2
+    else:
+        raise AssertionError("NaN accepted")
+
+
 # --------------------------------------------------------------------------- assignment
 def check_assign_worked_example(orc):
     """Sec. 3.2 example: D = 7/32; 37.5% -> m = 2, 18.75% -> m = 8."""
@@ -340,6 +411,7 @@ def check_gru_split_columns(orc):
 
 
 ALL_CHECKS = [
+    check_topk_worked_example, check_topk_random, check_topk_ties,
     check_assign_worked_example, check_assign_random, check_block_counts,
     check_pruning_ratio_identity, check_encode_random, check_encode_bf16,
     check_encode_special_values, check_encode_nan, check_product_exhaustive,

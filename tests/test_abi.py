@@ -102,6 +102,14 @@ def test_encode_allocation_failure_is_reported(L, monkeypatch):
     assert st == darb.ERR_OOM and h is None
 
 
+def test_assign_from_weights_allocation_failure_is_reported(L, monkeypatch):
+    monkeypatch.setenv("DARB_FAIL_ALLOC", "1")
+    nnz = np.zeros(4, np.int64)
+    m = np.zeros(4, np.int32)
+    assert L.darb_assign_from_weights(4096, darb.BF16, 4, 32, 32, 8, 1, 256, nnz.ctypes.data, m.ctypes.data,
+                                      None) == darb.ERR_OOM
+
+
 def test_calls_reject_unknown_handles(L):
     bogus = ctypes.c_void_p(0xDEAD0)
     info = darb._Info()
@@ -118,6 +126,24 @@ def test_calls_reject_unknown_handles(L):
     assert L.darb_rnn_reserve(bogus, 4) == darb.ERR_INVALID_ARG
     assert L.darb_destroy(bogus) == darb.ERR_INVALID_ARG
     assert L.darb_destroy(None) == darb.OK
+
+
+def test_assign_from_weights_rejects_bad_arguments_before_any_cuda_work(L):
+    nnz = np.zeros(4, np.int64)
+    m = np.zeros(4, np.int32)
+    call = lambda W, dt, rows, cols, ldw, keep, lo, hi, mo: L.darb_assign_from_weights(
+        W, dt, rows, cols, ldw, keep, lo, hi, nnz.ctypes.data, mo, None)
+    assert call(None, darb.BF16, 4, 8, 8, 4, 1, 256, m.ctypes.data) == darb.ERR_INVALID_ARG      # no W
+    assert call(4096, darb.BF16, 4, 8, 8, 4, 1, 256, None) == darb.ERR_INVALID_ARG               # no m_out
+    assert call(4096, 7, 4, 8, 8, 4, 1, 256, m.ctypes.data) == darb.ERR_INVALID_ARG              # dtype
+    assert call(4096, darb.BF16, 0, 8, 8, 4, 1, 256, m.ctypes.data) == darb.ERR_INVALID_ARG      # rows
+    assert call(4096, darb.BF16, 4, 8, 7, 4, 1, 256, m.ctypes.data) == darb.ERR_INVALID_ARG      # ldw < cols
+    assert call(4096, darb.BF16, 4, 8, 8, 0, 1, 256, m.ctypes.data) == darb.ERR_INVALID_ARG      # keep < 1
+    assert call(4096, darb.BF16, 4, 8, 8, 33, 1, 256, m.ctypes.data) == darb.ERR_INVALID_ARG     # keep > rows*cols
+    assert call(4096, darb.BF16, 4, 8, 8, 4, 0, 256, m.ctypes.data) == darb.ERR_INVALID_ARG      # m_min
+    assert call(4096, darb.BF16, 4, 8, 8, 4, 8, 4, m.ctypes.data) == darb.ERR_INVALID_ARG        # m_max < m_min
+    assert call(4097, darb.F32, 4, 8, 8, 4, 1, 256, m.ctypes.data) == darb.ERR_INVALID_ARG       # misaligned
+    assert call(4096, darb.BF16, 1 << 17, 1 << 16, 1 << 16, 4, 1, 256, m.ctypes.data) == darb.ERR_UNSUPPORTED
 
 
 def test_import_rejects_bad_arguments(L):

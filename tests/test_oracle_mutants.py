@@ -38,6 +38,10 @@ MUTANTS = {
     "gru_swaps_z": ("h_out[j * B + b] = (1.0 - zz) * nn + zz * h_prev[j * B + b];",
                     "h_out[j * B + b] = zz * nn + (1.0 - zz) * h_prev[j * B + b];"),
     "gru_split_off_by_one": ("if (k < I) {", "if (k <= I) {"),
+    "topk_strict_threshold": ("if (fabs(LOAD(W[r * ldw + c])) >= t) ++n;", "if (fabs(LOAD(W[r * ldw + c])) > t) ++n;"),
+    "topk_off_by_one_rank": ("const double t = mag[keep - 1];", "const double t = mag[keep < rows * cols ? keep : keep - 1];"),
+    "topk_ascending": ("return (x < y) - (x > y);", "return (x > y) - (x < y);"),
+    "topk_signed_values": ("mag[r * cols + c] = fabs(v);", "mag[r * cols + c] = v;"),
 }
 
 
