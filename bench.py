@@ -551,6 +551,27 @@ def run_rnn(torch, darb, synth, peak, reps=3):
 
             ms = seq_time(run, graph=True)
             ms_eager = seq_time(run, graph=False)
+
+            # the same layers, each as one persistent launch over all its steps
+            hseq = [torch.empty((wl.steps, H, B), device=dev) for _ in hs]
+            clast = [torch.empty((H, B), device=dev) for _ in hs]
+            zero = torch.zeros((H, B), device=dev)
+
+            def run_seq():
+                inp = xs
+                for li, (h, _) in enumerate(hs):
+                    if wl.kind == "lstm":
+                        darb.darb_lstm_sequence(h, wl.steps, I, H, B, inp, zero, zero, bias[li], hseq[li],
+                                                None, clast[li])
+                    else:
+                        darb.darb_gru_sequence(h, wl.steps, I, H, B, inp, zero, bias[li], bias2[li], hseq[li])
+                    inp = hseq[li]
+
+            try:
+                ms_seq = seq_time(run_seq, graph=False)
+            except darb.DarbError as e:
+                ms_seq = None
+                seq_note = str(e)
             nsteps = wl.steps * wl.layers
             us = ms * 1e3 / nsteps
             nbytes = sum(step_bytes(info, I, H, B, wl.kind) for _, info in hs) / wl.layers
@@ -559,7 +580,11 @@ def run_rnn(torch, darb, synth, peak, reps=3):
                                    "gflops": round(2 * sum(i["nnzb"] for _, i in hs) / wl.layers * B / (us * 1e-6) / 1e9, 1),
                                    "sequence_ms": round(ms, 3),
                                    "us_per_cell_step_eager": round(ms_eager * 1e3 / nsteps, 2),
-                                   "timing": "CUDA-graph replay of the whole sequence; eager: one Python call per step"}
+                                   "us_per_cell_step_persistent": (round(ms_seq * 1e3 / nsteps, 2)
+                                                                   if ms_seq is not None else seq_note),
+                                   "sequence_ms_persistent": round(ms_seq, 3) if ms_seq is not None else None,
+                                   "timing": "CUDA-graph replay of the whole sequence; eager: one Python call per "
+                                             "step; persistent: one darb_*_sequence launch per layer"}
         for h, _ in hs:
             darb.darb_destroy(h)
     return out

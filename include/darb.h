@@ -222,6 +222,48 @@ DARB_API darb_status_t darb_gru_step(darb_handle_t h, int64_t I, int64_t H, int6
                             float *h_out, cudaStream_t stream);
 
 /*
+ * T consecutive LSTM steps (the cell of darb_lstm_step) in one persistent
+ * launch: the recurrence of an RNN layer over a whole input sequence (the
+ * LSTM models of Sec. 4.1 run one step per token).  Each CTA keeps its share
+ * of the gate matrix decoded in shared memory for all T steps and the steps
+ * are separated by a grid-wide barrier, so W is read from memory once per
+ * call instead of once per step.
+ *   x_seq  device fp32, T x I x B (step t at x_seq + t*I*B); NULL allowed when I == 0
+ *   h0, c0 device fp32, H x B: the state before the first step
+ *   bias   device fp32 [4H] or NULL
+ *   h_seq  device fp32, T x H x B: h_t of every step
+ *   c_seq  device fp32, T x H x B: c_t of every step, or NULL
+ *   c_last device fp32, H x B: c_T, or NULL
+ * No output may overlap an input or another output.  T == 0 launches nothing
+ * and copies c0 to c_last.  The results equal T calls of darb_lstm_step up to
+ * the order of the fp32 additions inside each gate sum.
+ * Resources: one cooperative launch of one CTA per SM (at most H CTAs); a
+ * stream-ordered workspace of 256 bytes (plus H x B floats when c_last is
+ * NULL).  A barrier wait longer than 1 s ends the launch and is reported by
+ * darb_sync_status as DARB_ERR_TIMEOUT.
+ * Errors: DARB_ERR_INVALID_ARG (shape mismatch, null, overlap, T < 0);
+ * DARB_ERR_UNSUPPORTED when a CTA's share of the decoded matrix plus one
+ * column tile of [x_t; h_{t-1}] does not fit in shared memory, or cols > 65535;
+ * DARB_ERR_OOM; DARB_ERR_CUDA.
+ */
+DARB_API darb_status_t darb_lstm_sequence(darb_handle_t h, int64_t T, int64_t I, int64_t H, int64_t B,
+                                          const float *x_seq, const float *h0, const float *c0,
+                                          const float *bias, float *h_seq, float *c_seq, float *c_last,
+                                          cudaStream_t stream);
+
+/*
+ * T consecutive GRU steps (the cell of darb_gru_step) in one persistent
+ * launch, as darb_lstm_sequence.
+ *   x_seq device fp32, T x I x B (NULL allowed when I == 0); h0 device fp32
+ *   H x B; b_ih, b_hh device fp32 [3H] or NULL; h_seq device fp32, T x H x B,
+ *   not overlapping any input.
+ * Resources and errors as darb_lstm_sequence.
+ */
+DARB_API darb_status_t darb_gru_sequence(darb_handle_t h, int64_t T, int64_t I, int64_t H, int64_t B,
+                                         const float *x_seq, const float *h0, const float *b_ih,
+                                         const float *b_hh, float *h_seq, cudaStream_t stream);
+
+/*
  * darb_lstm_step without any allocation: the same step, same arguments and
  * same results, with its scratch (gate sums and arrival counters) in one
  * fixed array of 4 MiB inside this library instead of memory owned by the

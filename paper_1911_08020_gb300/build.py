@@ -19,7 +19,7 @@ INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libdarb.so")
 SOURCES = ["darb_api.cu", "assign.cu", "encode.cu", "spmm.cu", "spmm_batch.cu", "spmm_tc.cu", "rnn.cu", "rnn_batch.cu",
-           "noalloc.cu"]
+           "noalloc.cu", "sequence.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

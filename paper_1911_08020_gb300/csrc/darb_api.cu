@@ -633,6 +633,59 @@ darb_status_t darb_gru_step(darb_handle_t h, int64_t I, int64_t H, int64_t B, co
                                              sc, stream, early_ok(h, stream)));
 }
 
+// Arrival counts of the sequence kernels' barrier stay below 2^32.
+constexpr int64_t kMaxSequenceSteps = int64_t(1) << 22;
+
+static darb_status_t sequence_status(cudaError_t e) {
+    if (e == cudaErrorNotSupported) return DARB_ERR_UNSUPPORTED;
+    if (e == cudaErrorMemoryAllocation) return DARB_ERR_OOM;
+    return cuda_status(e);
+}
+
+darb_status_t darb_lstm_sequence(darb_handle_t h, int64_t T, int64_t I, int64_t H, int64_t B, const float *x_seq,
+                                 const float *h0, const float *c0, const float *bias, float *h_seq, float *c_seq,
+                                 float *c_last, cudaStream_t stream) {
+    // x_seq may be NULL when there are no steps
+    darb_status_t st = check_step(h, I, H, B, 4, T > 0 ? x_seq : h0, h0);
+    if (st != DARB_OK) return st;
+    if (T < 0 || c0 == nullptr || (T > 0 && h_seq == nullptr)) return DARB_ERR_INVALID_ARG;
+    if (T > kMaxSequenceSteps) return DARB_ERR_UNSUPPORTED;
+    const size_t hb = static_cast<size_t>(H * B) * 4, sb = hb * static_cast<size_t>(T);
+    const void *ins[4] = {x_seq, h0, c0, bias};
+    const size_t inb[4] = {static_cast<size_t>(I * B) * 4 * static_cast<size_t>(T), hb, hb,
+                           static_cast<size_t>(4 * H) * 4};
+    void *outs[3] = {h_seq, c_seq, c_last};
+    const size_t outb[3] = {sb, sb, hb};
+    for (int o = 0; o < 3; ++o) {
+        for (int i = 0; i < 4; ++i)
+            if (overlaps(outs[o], outb[o], ins[i], inb[i])) return DARB_ERR_INVALID_ARG;
+        for (int p = o + 1; p < 3; ++p)
+            if (overlaps(outs[o], outb[o], outs[p], outb[p])) return DARB_ERR_INVALID_ARG;
+    }
+    if (T == 0)
+        return c_last ? cuda_status(cudaMemcpyAsync(c_last, c0, hb, cudaMemcpyDeviceToDevice, stream)) : DARB_OK;
+    return sequence_status(darb::launch_lstm_sequence(format_of(h), h->row_m.data(), T, I, H, B, x_seq, h0, c0,
+                                                      bias, h_seq, c_seq, c_last, stream));
+}
+
+darb_status_t darb_gru_sequence(darb_handle_t h, int64_t T, int64_t I, int64_t H, int64_t B, const float *x_seq,
+                                const float *h0, const float *b_ih, const float *b_hh, float *h_seq,
+                                cudaStream_t stream) {
+    darb_status_t st = check_step(h, I, H, B, 3, T > 0 ? x_seq : h0, h0);
+    if (st != DARB_OK) return st;
+    if (T < 0 || (T > 0 && h_seq == nullptr)) return DARB_ERR_INVALID_ARG;
+    if (T > kMaxSequenceSteps) return DARB_ERR_UNSUPPORTED;
+    const size_t hb = static_cast<size_t>(H * B) * 4, sb = hb * static_cast<size_t>(T);
+    const void *ins[4] = {x_seq, h0, b_ih, b_hh};
+    const size_t inb[4] = {static_cast<size_t>(I * B) * 4 * static_cast<size_t>(T), hb,
+                           static_cast<size_t>(3 * H) * 4, static_cast<size_t>(3 * H) * 4};
+    for (int i = 0; i < 4; ++i)
+        if (overlaps(h_seq, sb, ins[i], inb[i])) return DARB_ERR_INVALID_ARG;
+    if (T == 0) return DARB_OK;
+    return sequence_status(darb::launch_gru_sequence(format_of(h), h->row_m.data(), T, I, H, B, x_seq, h0, b_ih,
+                                                     b_hh, h_seq, stream));
+}
+
 darb_status_t darb_info(darb_handle_t h, darb_info_t *info) {
     if (!live(h) || info == nullptr) return DARB_ERR_INVALID_ARG;
     darb_info_t r{};

@@ -129,6 +129,16 @@ cudaError_t launch_gru_step(const Format &f, int64_t I, int64_t H, int64_t B, co
                             const float *h_prev, const float *b_ih, const float *b_hh,
                             float *h_out, RnnScratch s, cudaStream_t stream, bool early = false);
 
+// T steps of an RNN layer in one persistent cooperative launch (sequence.cu).
+// row_m: the host copy of the per-row block sizes.  cudaErrorNotSupported
+// when a CTA's share of the matrix and one input tile do not fit on chip.
+cudaError_t launch_lstm_sequence(const Format &f, const int32_t *row_m, int64_t T, int64_t I, int64_t H, int64_t B,
+                                 const float *x, const float *h0, const float *c0, const float *bias, float *h_seq,
+                                 float *c_seq, float *c_last, cudaStream_t stream);
+cudaError_t launch_gru_sequence(const Format &f, const int32_t *row_m, int64_t T, int64_t I, int64_t H, int64_t B,
+                                const float *x, const float *h0, const float *b_ih, const float *b_hh, float *h_seq,
+                                cudaStream_t stream);
+
 struct RnnArgs;
 // Batch > 4 RNN steps (rnn_batch.cu); mode is kModeLstm or kModeGru.
 cudaError_t launch_rnn_batch(const Format &f, const RnnArgs &ra, int mode, bool early, cudaStream_t stream);

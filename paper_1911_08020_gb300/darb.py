@@ -62,6 +62,8 @@ def lib():
                 "darb_lstm_step": [P, I64, I64, I64, P, P, P, P, P, P, S],
                 "darb_lstm_step_noalloc": [P, I64, I64, I64, P, P, P, P, P, P, S],
                 "darb_gru_step": [P, I64, I64, I64, P, P, P, P, P, S],
+                "darb_lstm_sequence": [P, I64, I64, I64, I64, P, P, P, P, P, P, P, S],
+                "darb_gru_sequence": [P, I64, I64, I64, I64, P, P, P, P, P, S],
                 "darb_rnn_reserve": [P, I64],
                 "darb_info": [P, P],
                 "darb_export": [P, P, P, P, P],
@@ -244,6 +246,26 @@ def darb_gru_step(h: Handle, I: int, H: int, B: int, x, h_prev, b_ih, b_hh, h_ou
         _require_cuda_f32(t, n)
     _check(lib().darb_gru_step(h.ptr, I, H, B, _ptr(x), _ptr(h_prev), _ptr(b_ih), _ptr(b_hh),
                                _ptr(h_out), _stream(stream)), "darb_gru_step")
+
+
+def darb_lstm_sequence(h: Handle, T: int, I: int, H: int, B: int, x_seq, h0, c0, bias, h_seq,
+                       c_seq=None, c_last=None, stream=None):
+    """T LSTM steps in one persistent launch: x_seq (T, I, B) -> h_seq (T, H, B),
+    optionally every c_t (c_seq) and the last c (c_last)."""
+    for t, n in ((x_seq, "x_seq"), (h0, "h0"), (c0, "c0"), (bias, "bias"), (h_seq, "h_seq"),
+                 (c_seq, "c_seq"), (c_last, "c_last")):
+        _require_cuda_f32(t, n)
+    _check(lib().darb_lstm_sequence(h.ptr, T, I, H, B, _ptr(x_seq), _ptr(h0), _ptr(c0), _ptr(bias),
+                                    _ptr(h_seq), _ptr(c_seq), _ptr(c_last), _stream(stream)),
+           "darb_lstm_sequence")
+
+
+def darb_gru_sequence(h: Handle, T: int, I: int, H: int, B: int, x_seq, h0, b_ih, b_hh, h_seq, stream=None):
+    """T GRU steps in one persistent launch: x_seq (T, I, B) -> h_seq (T, H, B)."""
+    for t, n in ((x_seq, "x_seq"), (h0, "h0"), (b_ih, "b_ih"), (b_hh, "b_hh"), (h_seq, "h_seq")):
+        _require_cuda_f32(t, n)
+    _check(lib().darb_gru_sequence(h.ptr, T, I, H, B, _ptr(x_seq), _ptr(h0), _ptr(b_ih), _ptr(b_hh),
+                                   _ptr(h_seq), _stream(stream)), "darb_gru_sequence")
 
 
 def darb_rnn_reserve(h: Handle, max_batch: int):

@@ -121,6 +121,9 @@ def test_calls_reject_unknown_handles(L):
     assert L.darb_spmm_path(bogus, 256, ctypes.byref(pth), ctypes.byref(nk)) == darb.ERR_INVALID_ARG
     assert L.darb_lstm_step(bogus, 1, 1, 1, 4096, 4096, 4096, None, 8192, 8192, None) == darb.ERR_INVALID_ARG
     assert L.darb_gru_step(bogus, 1, 1, 1, 4096, 4096, None, None, 8192, None) == darb.ERR_INVALID_ARG
+    assert L.darb_lstm_sequence(bogus, 2, 1, 1, 1, 4096, 4096, 4096, None, 8192, None, None,
+                                None) == darb.ERR_INVALID_ARG
+    assert L.darb_gru_sequence(bogus, 2, 1, 1, 1, 4096, 4096, None, None, 8192, None) == darb.ERR_INVALID_ARG
     assert L.darb_export(bogus, None, None, None, None) == darb.ERR_INVALID_ARG
     assert L.darb_reencode(bogus, 4096, 8, None) == darb.ERR_INVALID_ARG
     assert L.darb_rnn_reserve(bogus, 4) == darb.ERR_INVALID_ARG
