@@ -24,8 +24,14 @@
  *    and any scratch it allocates, and releases both in darb_destroy.
  *  - Work is enqueued on the caller's stream.  Only darb_encode, darb_import,
  *    darb_export, darb_sync_status, darb_rnn_reserve and darb_destroy
- *    synchronise; the product and step calls are asynchronous and allocate
- *    nothing (except the RNN step scratch noted below).
+ *    synchronise; the product, step and sequence calls are asynchronous and
+ *    allocate nothing beyond the RNN step scratch and the pool scratch noted
+ *    below.
+ *  - Scratch that a call takes from the device's stream-ordered memory pool
+ *    (the tensor-core product, the sequence calls) is returned to the pool on
+ *    the same stream.  The first such call on a device raises the release
+ *    threshold of the device's current pool to 1 GiB if it is lower, so that
+ *    freed scratch stays mapped across synchronisations.
  *  - There is no CPU fallback: without a usable CUDA device the GPU calls
  *    return DARB_ERR_CUDA.
  */
@@ -237,10 +243,17 @@ DARB_API darb_status_t darb_gru_step(darb_handle_t h, int64_t I, int64_t H, int6
  * No output may overlap an input or another output.  T == 0 launches nothing
  * and copies c0 to c_last.  The results equal T calls of darb_lstm_step up to
  * the order of the fp32 additions inside each gate sum.
+ * When x_t is at least a third of the stacked input (2I >= H), the sequence
+ * has 64 to 2^19 columns (T * B) and the workspace below stays under 1 GiB,
+ * the x parts of all T steps are computed first as one product
+ * W [x_0 .. x_{T-1}; 0] of T * B columns (darb_spmm's kernels and numerics,
+ * the tensor cores for bf16 weights); the recurrence then stages and
+ * multiplies only h_{t-1}.
  * Resources: one cooperative launch of one CTA per SM (at most H CTAs); a
- * stream-ordered workspace of 256 bytes (plus H x B floats when c_last is
- * NULL).  A barrier wait longer than 1 s ends the launch and is reported by
- * darb_sync_status as DARB_ERR_TIMEOUT.
+ * stream-ordered workspace of 256 bytes, plus H x B floats when c_last is
+ * NULL and the cell state does not fit on chip, plus (I + H + 4H) x T*B
+ * floats when the x parts are precomputed.  A barrier wait longer than 1 s
+ * ends the launch and is reported by darb_sync_status as DARB_ERR_TIMEOUT.
  * Errors: DARB_ERR_INVALID_ARG (shape mismatch, null, overlap, T < 0);
  * DARB_ERR_UNSUPPORTED when a CTA's share of the decoded matrix plus one
  * column tile of [x_t; h_{t-1}] does not fit in shared memory, or cols > 65535;
@@ -257,7 +270,8 @@ DARB_API darb_status_t darb_lstm_sequence(darb_handle_t h, int64_t T, int64_t I,
  *   x_seq device fp32, T x I x B (NULL allowed when I == 0); h0 device fp32
  *   H x B; b_ih, b_hh device fp32 [3H] or NULL; h_seq device fp32, T x H x B,
  *   not overlapping any input.
- * Resources and errors as darb_lstm_sequence.
+ * Precomputed x parts, resources and errors as darb_lstm_sequence (workspace
+ * with 3H rows of x parts).
  */
 DARB_API darb_status_t darb_gru_sequence(darb_handle_t h, int64_t T, int64_t I, int64_t H, int64_t B,
                                          const float *x_seq, const float *h0, const float *b_ih,

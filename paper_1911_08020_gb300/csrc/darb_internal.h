@@ -149,6 +149,14 @@ int rnn_batch_tile(int64_t B);
 // Streaming multiprocessors of the current device (cached).
 int sm_count();
 
+// Stream-ordered scratch (cudaMallocAsync).  The first call on a device raises
+// the release threshold of the device's current memory pool to kPoolKeep (it
+// never lowers it): scratch freed before a synchronisation then stays mapped
+// for the next call instead of being unmapped at the synchronisation and mapped
+// again, which costs more than the kernels the scratch serves.
+constexpr uint64_t kPoolKeep = uint64_t(1) << 30;
+cudaError_t stream_alloc(void **p, size_t bytes, cudaStream_t stream);
+
 // Row densities of Sec. 3.2's first step (assign.cu): row_nnz[r] = number of
 // weights of row r whose magnitude is >= the keep-th largest magnitude of W.
 // work: 4608 bytes of device scratch; nan_flag: device int, set if W has a NaN.

@@ -29,11 +29,12 @@
 namespace darb {
 namespace seq {
 
-constexpr int kThreads = 256;
+constexpr int kThreads = 512;
 constexpr int kSeqWarps = kThreads / 32;
 constexpr int kMaxCtas = 256;
 constexpr size_t kSmemCap = 226 * 1024;   // dynamic shared memory, below the 227 KB opt-in with room for the static part
-constexpr int kMaxTile = 32;   // batch columns per tile, at most (one per lane)
+constexpr int kMaxTile = 32;              // batch columns per tile, at most (one per lane)
+constexpr size_t kCellOnChip = 16 * 1024; // LSTM cell state kept in shared memory up to this size
 
 struct Ranges {
     int32_t start[kMaxCtas + 1];   // CTA q owns hidden units [start[q], start[q+1])
@@ -43,7 +44,12 @@ struct SeqArgs {
     int I, H, T;
     int lbt;                // log2 of the batch tile width bt (bt <= 32)
     int stage_mode;         // kStage*
+    int piece;              // kept weights per work item, at most
+    int c_on_chip;          // LSTM: cell state in shared memory
     int64_t B;
+    const float *gx;        // x parts of the gate sums of every step, rows x ldgx (row r, step t, column b
+                            // at r * ldgx + t * B + b), or nullptr: x_t is staged with h_{t-1} instead
+    int64_t ldgx;
     const float *x;         // T x I x B
     const float *h0;        // H x B
     const float *c0;        // H x B (LSTM)
@@ -52,7 +58,8 @@ struct SeqArgs {
     const float *b_hh;      // GRU [3H] or nullptr
     float *h_seq;           // T x H x B
     float *c_seq;           // T x H x B or nullptr (LSTM)
-    float *c_state;         // H x B: the running cell state (LSTM)
+    float *c_state;         // H x B: the running cell state when it is not on chip (LSTM)
+    float *c_last;          // H x B or nullptr (LSTM)
     unsigned *bar;          // arrival counter, zero at launch
     int *abort_flag;        // zero at launch
     int32_t *status;
@@ -60,26 +67,30 @@ struct SeqArgs {
 
 // Byte offsets of the regions of a CTA's dynamic shared memory.
 struct SmemPlan {
-    uint32_t w_off, rowptr_off, mid_off, sorted_off, cnt_off, in_off, gate_off, total;
-    int rows_cap;
+    uint32_t w_off, rowptr_off, mid_off, rowitem_off, item_off, bias_off, c_off, gx_off, in_off, part_off, total;
+    int items_cap;
 };
 
-inline SmemPlan smem_plan(int kept_cap, int rows_cap, bool bf16, bool gru, int in_rows, int bt) {
+inline SmemPlan smem_plan(int64_t kept_cap, int rows_cap, int items_cap, int units_cap, bool bf16, bool gru,
+                          int in_rows, int bt, int64_t B, bool c_on_chip, bool pre) {
     SmemPlan p{};
-    p.rows_cap = rows_cap;
+    p.items_cap = items_cap;
     size_t o = 0;
     auto take = [&](size_t bytes) {
         const size_t at = o;
         o = (o + bytes + 15) / 16 * 16;
-        return static_cast<uint32_t>(at);
+        return static_cast<uint32_t>(std::min<size_t>(at, UINT32_MAX));
     };
     p.w_off = take(size_t(kept_cap) * (bf16 ? 4 : 8));
     p.rowptr_off = take(size_t(rows_cap + 1) * 4);
     p.mid_off = take(size_t(rows_cap) * 4);
-    p.sorted_off = take(size_t(rows_cap) * 4);
-    p.cnt_off = take(size_t(rows_cap) * 4);
+    p.rowitem_off = take(size_t(rows_cap + 1) * 4);
+    p.item_off = take(size_t(items_cap) * 16);
+    p.bias_off = take(size_t(rows_cap) * 2 * 4);
+    p.c_off = take(c_on_chip ? size_t(units_cap) * size_t(B) * 4 : 0);
+    p.gx_off = take(pre ? size_t(rows_cap) * bt * 4 : 0);
     p.in_off = take(size_t(in_rows) * bt * 4);
-    p.gate_off = take(size_t(gru ? 2 : 1) * rows_cap * bt * 4);
+    p.part_off = take(size_t(gru ? 2 : 1) * items_cap * bt * 4);
     p.total = static_cast<uint32_t>(std::min<size_t>(o, UINT32_MAX));
     return p;
 }
@@ -133,49 +144,86 @@ __device__ __forceinline__ bool grid_barrier(const SeqArgs &a, unsigned target, 
     return *s_ok != 0;
 }
 
+// Sum over kept weights [pa, pb) of the CTA, subgroup `sub` taking every S-th
+// weight from pa + sub, against batch column `col` of the staged input.
+template <class P>
+__device__ __forceinline__ float dot_range(const typename P::T *s_w, const float *s_in, int pa, int pb, int sub, int S,
+                                           int lbt, int col) {
+    float acc0 = 0.0f, acc1 = 0.0f;
+    int p = pa + sub;
+    for (; p + 3 * S < pb; p += 4 * S) {
+        const typename P::T w0 = s_w[p], w1 = s_w[p + S], w2 = s_w[p + 2 * S], w3 = s_w[p + 3 * S];
+        const float v0 = s_in[(P::col(w0) << lbt) + col], v1 = s_in[(P::col(w1) << lbt) + col];
+        const float v2 = s_in[(P::col(w2) << lbt) + col], v3 = s_in[(P::col(w3) << lbt) + col];
+        acc0 = fmaf(P::val(w0), v0, acc0);
+        acc1 = fmaf(P::val(w1), v1, acc1);
+        acc0 = fmaf(P::val(w2), v2, acc0);
+        acc1 = fmaf(P::val(w3), v3, acc1);
+    }
+    for (; p < pb; p += S) {
+        const typename P::T w = s_w[p];
+        acc0 = fmaf(P::val(w), s_in[(P::col(w) << lbt) + col], acc0);
+    }
+    return acc0 + acc1;
+}
+
 // Input staging modes, chosen on the host from the shapes and alignments.
 constexpr int kStageScalar = 0;   // one float per load
 constexpr int kStageQuadCols = 1; // 4 batch columns per 16-byte load (B and bt multiples of 4, aligned)
 constexpr int kStageQuadRows = 2; // B == 1: 4 input rows per 16-byte load (I, H multiples of 4, aligned)
 constexpr int kStageUnroll = 8;   // loads a thread has in flight
 
-// s_in[k][j] = [x_t; h_{t-1}][k][b0 + j] for j < nb, 0 for nb <= j < bt.
+// s_in[k][j] = [x_t; h_{t-1}][k][b0 + j] for j < nb, 0 for nb <= j < bt, for
+// the K staged rows, of which the first I come from x_t (I = 0: h only).
 // h_{t-1} was written by other CTAs of this launch, so every load goes to L2
 // (ld.cg); the loads of a thread are issued together so that enough bytes are
-// in flight to cover the L2 latency.
-__device__ __forceinline__ void stage_input(const SeqArgs &a, const float *xt, const float *hp, int64_t b0, int nb,
-                                            float *s_in) {
-    const int I = a.I, K = a.I + a.H, lbt = a.lbt, bt = 1 << lbt;
+// in flight to cover the L2 latency, and each CTA starts its sweep at its own
+// offset so that the CTAs do not all ask for the same lines at once.
+__device__ __forceinline__ void stage_input(const SeqArgs &a, int I, int K, const float *xt, const float *hp,
+                                            int64_t b0, int nb, float *s_in) {
+    const int lbt = a.lbt, bt = 1 << lbt;
     const int64_t B = a.B;
     const int tid = threadIdx.x;
     auto src = [&](int k) { return k < I ? xt + int64_t(k) * B : hp + int64_t(k - I) * B; };
     if (a.stage_mode == kStageQuadCols) {
         const int lq = lbt - 2, n = K << lq;   // quads
+        const int rot = static_cast<int>(int64_t(blockIdx.x) * n / gridDim.x);
         for (int i0 = tid; i0 < n; i0 += kThreads * kStageUnroll) {
             float4 v[kStageUnroll];
 #pragma unroll
             for (int u = 0; u < kStageUnroll; ++u) {
-                const int i = i0 + u * kThreads;
-                const int k = i >> lq, j = (i & ((1 << lq) - 1)) * 4;
+                int i = i0 + u * kThreads;
                 v[u] = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
-                if (i < n && j < nb) v[u] = __ldcg(reinterpret_cast<const float4 *>(src(k) + b0 + j));
+                if (i < n) {
+                    i = i + rot < n ? i + rot : i + rot - n;
+                    const int k = i >> lq, j = (i & ((1 << lq) - 1)) * 4;
+                    if (j < nb) v[u] = __ldcg(reinterpret_cast<const float4 *>(src(k) + b0 + j));
+                }
             }
 #pragma unroll
-            for (int u = 0; u < kStageUnroll; ++u)
-                if (i0 + u * kThreads < n) reinterpret_cast<float4 *>(s_in)[i0 + u * kThreads] = v[u];
+            for (int u = 0; u < kStageUnroll; ++u) {
+                const int i = i0 + u * kThreads;
+                if (i < n) reinterpret_cast<float4 *>(s_in)[i + rot < n ? i + rot : i + rot - n] = v[u];
+            }
         }
     } else if (a.stage_mode == kStageQuadRows) {
         const int n = K >> 2;
+        const int rot = static_cast<int>(int64_t(blockIdx.x) * n / gridDim.x);
         for (int i0 = tid; i0 < n; i0 += kThreads * kStageUnroll) {
             float4 v[kStageUnroll];
 #pragma unroll
             for (int u = 0; u < kStageUnroll; ++u) {
-                const int i = i0 + u * kThreads;
-                if (i < n) v[u] = __ldcg(reinterpret_cast<const float4 *>(src(4 * i)));
+                int i = i0 + u * kThreads;
+                if (i < n) {
+                    i = i + rot < n ? i + rot : i + rot - n;
+                    v[u] = __ldcg(reinterpret_cast<const float4 *>(src(4 * i)));
+                }
             }
 #pragma unroll
-            for (int u = 0; u < kStageUnroll; ++u)
-                if (i0 + u * kThreads < n) reinterpret_cast<float4 *>(s_in)[i0 + u * kThreads] = v[u];
+            for (int u = 0; u < kStageUnroll; ++u) {
+                const int i = i0 + u * kThreads;
+                if (i < n) reinterpret_cast<float4 *>(s_in)[i + rot < n ? i + rot : i + rot - n] = v[u];
+            }
         }
     } else {
         const int n = K << lbt;
@@ -203,14 +251,17 @@ seq_kernel(Format f, SeqArgs a, Ranges rg, SmemPlan sp) {
     using P = Packed<BF16>;
     using PT = typename P::T;
     extern __shared__ __align__(16) unsigned char sm[];
-    __shared__ int s_ok;
+    __shared__ int s_ok, s_nitems;
     PT *s_w = reinterpret_cast<PT *>(sm + sp.w_off);
     int *s_rowptr = reinterpret_cast<int *>(sm + sp.rowptr_off);
-    int *s_mid = reinterpret_cast<int *>(sm + sp.mid_off);        // GRU: first kept weight on h
-    int *s_sorted = reinterpret_cast<int *>(sm + sp.sorted_off);  // local rows, most weights first
-    int *s_cnt = reinterpret_cast<int *>(sm + sp.cnt_off);
-    float *s_in = reinterpret_cast<float *>(sm + sp.in_off);      // [I + H][bt]
-    float *s_gate = reinterpret_cast<float *>(sm + sp.gate_off);  // [parts][R][bt]
+    int *s_mid = reinterpret_cast<int *>(sm + sp.mid_off);          // GRU: first kept weight of a row on h
+    int *s_rowitem = reinterpret_cast<int *>(sm + sp.rowitem_off);  // items of local row lr: [s_rowitem[lr], s_rowitem[lr+1])
+    int4 *s_item = reinterpret_cast<int4 *>(sm + sp.item_off);      // (first, end, local row, first on h)
+    float *s_bias = reinterpret_cast<float *>(sm + sp.bias_off);    // [R] (GRU: [2R], b_ih then b_hh)
+    float *s_c = reinterpret_cast<float *>(sm + sp.c_off);          // [units][B] when on chip
+    float *s_gx = reinterpret_cast<float *>(sm + sp.gx_off);        // [R][bt]: x parts of this tile
+    float *s_in = reinterpret_cast<float *>(sm + sp.in_off);        // [kin + 1][bt], last row zero
+    float *s_part = reinterpret_cast<float *>(sm + sp.part_off);    // [parts][items][bt]
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int u0 = rg.start[blockIdx.x], nu = rg.start[blockIdx.x + 1] - u0;
     const int R = kGates * nu;   // local row q*nu + i is matrix row q*H + u0 + i
@@ -218,33 +269,54 @@ seq_kernel(Format f, SeqArgs a, Ranges rg, SmemPlan sp) {
     const int lbt = a.lbt, bt = 1 << lbt, S = 32 >> lbt;
     const int sub = lane >> lbt, col = lane & (bt - 1);
     const int64_t B = a.B;
+    // with the x parts precomputed only h_{t-1} is staged and only the kept
+    // weights of blocks that reach column I are kept on chip (columns shifted by I)
+    const bool pre = a.gx != nullptr;
+    const int kin = pre ? H : I + H, ioff = pre ? I : 0;
     auto grow = [&](int lr) { return (lr / nu) * H + u0 + lr % nu; };
 
-    // ---- prologue: weights per row, row pointers, rows by descending weight count
-    for (int lr = tid; lr < R; lr += kThreads) s_cnt[lr] = f.groups[f.rowloc[grow(lr)] / kSlots].n;
+    // ---- prologue: row sizes, biases, cell state, the zero row of the staged input
+    for (int lr = tid; lr < R; lr += kThreads) {
+        const int r = grow(lr);
+        const Group &g = f.groups[f.rowloc[r] / kSlots];
+        s_rowptr[lr + 1] = g.n - (pre ? I / g.m : 0);
+        if constexpr (kGru) {
+            s_bias[lr] = a.b_ih ? a.b_ih[r] : 0.0f;
+            s_bias[R + lr] = a.b_hh ? a.b_hh[r] : 0.0f;
+        } else {
+            s_bias[lr] = a.bias ? a.bias[r] : 0.0f;
+        }
+    }
+    if constexpr (!kGru)
+        if (a.c_on_chip)
+            for (int i = tid; i < nu * B; i += kThreads) s_c[i] = a.c0[int64_t(u0) * B + i];
+    for (int j = tid; j < bt; j += kThreads) s_in[(kin << lbt) + j] = 0.0f;
     __syncthreads();
+    // row pointers and work items: every row cut into pieces of at most a.piece weights
     if (tid == 0) {
-        int p = 0;
+        int p = 0, ni = 0;
         for (int lr = 0; lr < R; ++lr) {
+            const int n = s_rowptr[lr + 1];
             s_rowptr[lr] = p;
-            p += s_cnt[lr];
+            s_rowitem[lr] = ni;
+            for (int q = 0; q < n; q += a.piece) s_item[ni++] = make_int4(p + q, p + min(n, q + a.piece), lr, 0);
+            p += n;
         }
         s_rowptr[R] = p;
-    }
-    for (int lr = tid; lr < R; lr += kThreads) {
-        int rank = 0;
-        const int n = s_cnt[lr];
-        for (int l = 0; l < R; ++l) rank += (s_cnt[l] > n || (s_cnt[l] == n && l < lr)) ? 1 : 0;
-        s_sorted[rank] = lr;
+        s_rowitem[R] = ni;
+        s_nitems = ni;
     }
     __syncthreads();
+    // every kept weight as (value, column); a row's weights are in column order
     for (int lr = warp; lr < R; lr += kSeqWarps) {
         const int loc = f.rowloc[grow(lr)];
         const Group g = f.groups[loc / kSlots];
         const int slot = loc % kSlots;
         const int base = s_rowptr[lr];
         const int jmid = I / g.m;   // the only block that can hold columns on both sides of I
-        for (int j = lane; j < g.n; j += 32) {
+        const int jlo = pre ? jmid : 0;
+        if (pre && lane == 0) s_mid[lr] = base;   // everything kept here multiplies h
+        for (int j = jlo + lane; j < g.n; j += 32) {
             const int64_t rec = int64_t(j / kChunk) * kSlots + slot;
             const int q = j % kChunk;
             uint32_t bits;
@@ -253,107 +325,98 @@ seq_kernel(Format f, SeqArgs a, Ranges rg, SmemPlan sp) {
             uint32_t o;
             if (g.nib) o = (f.offs[g.off_off + rec] >> (4 * q)) & 15u;
             else o = (f.offs[g.off_off + 2 * rec + (q >> 2)] >> (8 * (q & 3))) & 255u;
-            const uint32_t c = uint32_t(j) * uint32_t(g.m) + o;
-            s_w[base + j] = P::make(bits, c);
-            if (j == jmid) s_mid[lr] = base + j + (c < uint32_t(I) ? 1 : 0);
+            uint32_t c = uint32_t(j) * uint32_t(g.m) + o;
+            if (pre) {
+                if (c < uint32_t(I)) {   // an x weight of the straddling block: its product is in gx
+                    bits = 0;
+                    c = uint32_t(kin);
+                } else {
+                    c -= uint32_t(ioff);
+                }
+            } else if (j == jmid) {
+                s_mid[lr] = base + j + (c < uint32_t(I) ? 1 : 0);
+            }
+            s_w[base + j - jlo] = P::make(bits, c);
         }
+    }
+    __syncthreads();
+    const int NI = s_nitems;
+    for (int i = tid; i < NI; i += kThreads) {
+        int4 it = s_item[i];
+        it.w = kGru ? max(it.x, min(it.y, s_mid[it.z])) : it.y;
+        s_item[i] = it;
     }
     __syncthreads();
 
     // ---- the steps
-    float *c_state = kGru ? nullptr : a.c_state + int64_t(u0) * B;
+    float *c_run = kGru ? nullptr : (a.c_on_chip ? s_c : a.c_state + int64_t(u0) * B);
     for (int t = 0; t < a.T; ++t) {
         const float *xt = a.x + int64_t(t) * I * B;
         const float *hp = t == 0 ? a.h0 : a.h_seq + int64_t(t - 1) * H * B;
         float *ht = a.h_seq + int64_t(t) * H * B + int64_t(u0) * B;
         float *ct = a.c_seq ? a.c_seq + int64_t(t) * H * B + int64_t(u0) * B : nullptr;
-        const float *cp = kGru ? nullptr : (t == 0 ? a.c0 + int64_t(u0) * B : c_state);
+        const float *cp = kGru ? nullptr : (t == 0 && !a.c_on_chip ? a.c0 + int64_t(u0) * B : c_run);
         for (int64_t b0 = 0; b0 < B; b0 += bt) {
             const int nb = static_cast<int>(B - b0 < bt ? B - b0 : bt);
-            // stage [x_t; h_{t-1}] for columns [b0, b0 + nb), zeros past the batch
-            stage_input(a, xt, hp, b0, nb, s_in);
+            // stage [x_t; h_{t-1}] (or h_{t-1}) for columns [b0, b0 + nb), zeros past the batch
+            if (pre)
+                for (int i = tid; i < R << lbt; i += kThreads) {
+                    const int lr = i >> lbt, j = i & (bt - 1);
+                    s_gx[i] = j < nb ? __ldg(a.gx + int64_t(grow(lr)) * a.ldgx + int64_t(t) * B + b0 + j) : 0.0f;
+                }
+            stage_input(a, pre ? 0 : I, kin, xt, hp, b0, nb, s_in);
             __syncthreads();
-            // gate sums; rows go to warps in a snake over the sorted order
-            for (int r0 = 0; r0 < R; r0 += kSeqWarps) {
-                const int round = r0 / kSeqWarps;
-                const int si = r0 + ((round & 1) ? kSeqWarps - 1 - warp : warp);
-                if (si >= R) continue;
-                const int lr = s_sorted[si];
-                const int p0 = s_rowptr[lr], p1 = s_rowptr[lr + 1];
-                const int pm = kGru ? s_mid[lr] : p1;
-                float ax = 0.0f, ah = 0.0f;
-                int p = p0 + sub;
-                for (; p + 3 * S < pm; p += 4 * S) {
-                    const PT w0 = s_w[p], w1 = s_w[p + S], w2 = s_w[p + 2 * S], w3 = s_w[p + 3 * S];
-                    const float v0 = s_in[(P::col(w0) << lbt) + col], v1 = s_in[(P::col(w1) << lbt) + col];
-                    const float v2 = s_in[(P::col(w2) << lbt) + col], v3 = s_in[(P::col(w3) << lbt) + col];
-                    ax = fmaf(P::val(w0), v0, ax);
-                    ax = fmaf(P::val(w1), v1, ax);
-                    ax = fmaf(P::val(w2), v2, ax);
-                    ax = fmaf(P::val(w3), v3, ax);
-                }
-                for (; p < pm; p += S) {
-                    const PT w = s_w[p];
-                    ax = fmaf(P::val(w), s_in[(P::col(w) << lbt) + col], ax);
-                }
-                if constexpr (kGru) {
-                    // the h part starts at pm; each subgroup keeps its stride from there
-                    p = pm + sub;
-                    for (; p + 3 * S < p1; p += 4 * S) {
-                        const PT w0 = s_w[p], w1 = s_w[p + S], w2 = s_w[p + 2 * S], w3 = s_w[p + 3 * S];
-                        const float v0 = s_in[(P::col(w0) << lbt) + col], v1 = s_in[(P::col(w1) << lbt) + col];
-                        const float v2 = s_in[(P::col(w2) << lbt) + col], v3 = s_in[(P::col(w3) << lbt) + col];
-                        ah = fmaf(P::val(w0), v0, ah);
-                        ah = fmaf(P::val(w1), v1, ah);
-                        ah = fmaf(P::val(w2), v2, ah);
-                        ah = fmaf(P::val(w3), v3, ah);
-                    }
-                    for (; p < p1; p += S) {
-                        const PT w = s_w[p];
-                        ah = fmaf(P::val(w), s_in[(P::col(w) << lbt) + col], ah);
-                    }
-                }
+            // partial gate sums of the work items; items go to warps in a snake
+            for (int r0 = 0; r0 < NI; r0 += kSeqWarps) {
+                const int ii = r0 + (((r0 / kSeqWarps) & 1) ? kSeqWarps - 1 - warp : warp);
+                if (ii >= NI) continue;
+                const int4 it = s_item[ii];
+                float ax = dot_range<P>(s_w, s_in, it.x, it.w, sub, S, lbt, col);
+                float ah = 0.0f;
+                if constexpr (kGru) ah = dot_range<P>(s_w, s_in, it.w, it.y, sub, S, lbt, col);
                 for (int o = 16; o >= bt; o >>= 1) {
                     ax += __shfl_xor_sync(0xFFFFFFFFu, ax, o);
                     if constexpr (kGru) ah += __shfl_xor_sync(0xFFFFFFFFu, ah, o);
                 }
                 if (sub == 0) {
-                    s_gate[(lr << lbt) + col] = ax;
-                    if constexpr (kGru) s_gate[((R + lr) << lbt) + col] = ah;
+                    s_part[(ii << lbt) + col] = ax;
+                    if constexpr (kGru) s_part[((NI + ii) << lbt) + col] = ah;
                 }
             }
             __syncthreads();
             // the cells of the owned units for these columns
+            auto gate = [&](int lr, int part, int j) {
+                float v = s_bias[part * R + lr];
+                for (int ii = s_rowitem[lr]; ii < s_rowitem[lr + 1]; ++ii) v += s_part[((part * NI + ii) << lbt) + j];
+                return v;
+            };
             for (int i = tid; i < nu << lbt; i += kThreads) {
-                const int ui = i >> lbt, j = i & (bt - 1), u = u0 + ui;
+                const int ui = i >> lbt, j = i & (bt - 1);
                 if (j >= nb) continue;
                 const int64_t e = int64_t(ui) * B + b0 + j;
+                auto xg = [&](int lr) { return pre ? s_gx[(lr << lbt) + j] : 0.0f; };
                 if constexpr (MODE == kModeLstm) {
-                    float pre[4];
-#pragma unroll
-                    for (int q = 0; q < 4; ++q)
-                        pre[q] = s_gate[((q * nu + ui) << lbt) + j] + (a.bias ? a.bias[q * H + u] : 0.0f);
-                    const float c = sigm(pre[1]) * cp[e] + sigm(pre[0]) * tanhf(pre[2]);
-                    c_state[e] = c;
+                    const float pi = gate(ui, 0, j) + xg(ui), pf = gate(nu + ui, 0, j) + xg(nu + ui);
+                    const float pg = gate(2 * nu + ui, 0, j) + xg(2 * nu + ui);
+                    const float po = gate(3 * nu + ui, 0, j) + xg(3 * nu + ui);
+                    const float c = sigm(pf) * cp[e] + sigm(pi) * tanhf(pg);
+                    c_run[e] = c;
                     if (ct) ct[e] = c;
-                    ht[e] = sigm(pre[3]) * tanhf(c);
+                    ht[e] = sigm(po) * tanhf(c);
                 } else {
-                    float ax[3], bh[3];
-#pragma unroll
-                    for (int q = 0; q < 3; ++q) {
-                        ax[q] = s_gate[((q * nu + ui) << lbt) + j] + (a.b_ih ? a.b_ih[q * H + u] : 0.0f);
-                        bh[q] = s_gate[((R + q * nu + ui) << lbt) + j] + (a.b_hh ? a.b_hh[q * H + u] : 0.0f);
-                    }
-                    const float rr = sigm(ax[0] + bh[0]);
-                    const float zz = sigm(ax[1] + bh[1]);
-                    const float nn = tanhf(ax[2] + rr * bh[2]);
-                    ht[e] = (1.0f - zz) * nn + zz * s_in[((I + u) << lbt) + j];
+                    const float rr = sigm(gate(ui, 0, j) + xg(ui) + gate(ui, 1, j));
+                    const float zz = sigm(gate(nu + ui, 0, j) + xg(nu + ui) + gate(nu + ui, 1, j));
+                    const float nn = tanhf(gate(2 * nu + ui, 0, j) + xg(2 * nu + ui) + rr * gate(2 * nu + ui, 1, j));
+                    ht[e] = (1.0f - zz) * nn + zz * s_in[((kin - H + u0 + ui) << lbt) + j];
                 }
             }
             __syncthreads();
         }
         if (t + 1 < a.T && !grid_barrier(a, unsigned(t + 1) * gridDim.x, &s_ok)) return;
     }
+    if constexpr (!kGru)
+        if (a.c_on_chip && a.c_last)
+            for (int i = tid; i < nu * B; i += kThreads) a.c_last[int64_t(u0) * B + i] = s_c[i];
 }
 
 }  // namespace seq
@@ -385,6 +448,27 @@ void split_units(const std::vector<int64_t> &kept, int G, seq::Ranges &rg, int64
 
 }  // namespace
 
+// x_t of every step laid out as the columns of one product input:
+// xall[k][t * B + b] = x[t][k][b] for k < I (a warp per (t, k), lanes over b).
+__global__ void __launch_bounds__(256) gather_x_kernel(const float *x, int T, int I, int64_t B, float *xall,
+                                                       int64_t ldx) {
+    const int lane = threadIdx.x & 31;
+    const int64_t nrows = int64_t(T) * I;
+    for (int64_t row = int64_t(blockIdx.x) * 8 + (threadIdx.x >> 5); row < nrows; row += int64_t(gridDim.x) * 8) {
+        const int64_t t = row / I, k = row % I;
+        const float *src = x + row * B;
+        float *dst = xall + k * ldx + t * B;
+        for (int64_t b = lane; b < B; b += 32) dst[b] = __ldg(src + b);
+    }
+}
+
+// Whether the x parts of all steps go through one darb_spmm-style product up
+// front: when x_t is a large share of the stacked input the per-step staging
+// and gate sums shrink by that share; the product has T*B columns.
+inline bool precompute_x(int64_t T, int64_t I, int64_t H, int64_t B, size_t ws_bytes) {
+    return I > 0 && 2 * I >= H && T * B >= 64 && T * B <= (int64_t(1) << 19) && ws_bytes <= (size_t(1) << 30);
+}
+
 template <bool BF16, int MODE>
 static cudaError_t launch_seq_t(const Format &f, const int32_t *row_m, seq::SeqArgs a, float *c_last,
                                 cudaStream_t stream) {
@@ -392,14 +476,21 @@ static cudaError_t launch_seq_t(const Format &f, const int32_t *row_m, seq::SeqA
     constexpr int kGates = MODE == kModeLstm ? 4 : 3;
     constexpr bool kGru = MODE == kModeGru;
     const int H = a.H, I = a.I;
+    const int64_t B = a.B, T = a.T, rows = f.rows;
     if (f.cols > 65535) return cudaErrorNotSupported;   // columns are kept in 16 bits
+    auto up = [](size_t v) { return (v + 255) / 256 * 256; };
+    const int64_t ldx = (T * B + 3) / 4 * 4;   // 16-byte rows for the product's loads
+    const size_t pre_bytes = up(size_t(I + H) * ldx * 4) + up(size_t(rows) * ldx * 4);
+    const bool pre = precompute_x(T, I, H, B, pre_bytes);
+    // kept weights on chip per row: all, or those of the blocks that reach column I
+    auto row_kept = [&](int64_t r) {
+        const int64_t m = row_m[r];
+        return (f.cols + m - 1) / m - (pre ? I / m : 0);
+    };
     std::vector<int64_t> kept(static_cast<size_t>(H));
     for (int u = 0; u < H; ++u) {
         int64_t k = 0;
-        for (int q = 0; q < kGates; ++q) {
-            const int64_t m = row_m[static_cast<size_t>(q) * H + u];
-            k += (f.cols + m - 1) / m;
-        }
+        for (int q = 0; q < kGates; ++q) k += row_kept(int64_t(q) * H + u);
         kept[static_cast<size_t>(u)] = k;
     }
     const int G = std::max(1, std::min({sm_count(), H, kMaxCtas}));
@@ -408,35 +499,71 @@ static cudaError_t launch_seq_t(const Format &f, const int32_t *row_m, seq::SeqA
     int units_cap = 0;
     split_units(kept, G, rg, kept_cap, units_cap);
     if (kept_cap > (int64_t(1) << 20)) return cudaErrorNotSupported;
-    // widest batch tile (a power of two, <= 32) whose staging still fits
+    const bool c_on_chip = !kGru && size_t(units_cap) * size_t(B) * 4 <= kCellOnChip;
+    const int kin = pre ? H : I + H;
+    // widest batch tile (a power of two, <= 32) whose staging still fits; rows
+    // are cut into work items of about kept_cap / (2 * warps) weights, and of at
+    // least 8 weights per lane of a subgroup
     int bt = 1;
-    while (bt < kMaxTile && bt < a.B) bt *= 2;
+    while (bt < kMaxTile && bt < B) bt *= 2;
     SmemPlan sp{};
+    int piece = 0;
     for (;; bt /= 2) {
-        sp = smem_plan(static_cast<int>(kept_cap), kGates * units_cap, BF16, kGru, I + H, bt);
+        const int S = kMaxTile / bt;
+        piece = static_cast<int>(std::max<int64_t>(8 * S, (kept_cap + 2 * kSeqWarps - 1) / (2 * kSeqWarps)));
+        int items_cap = 0;
+        for (int q = 0; q < G; ++q) {
+            int items = 0;
+            for (int g = 0; g < kGates; ++g)
+                for (int u = rg.start[q]; u < rg.start[q + 1]; ++u)
+                    items += static_cast<int>((row_kept(int64_t(g) * H + u) + piece - 1) / piece);
+            items_cap = std::max(items_cap, items);
+        }
+        sp = smem_plan(kept_cap, kGates * units_cap, items_cap, units_cap, BF16, kGru, kin + 1, bt, B, c_on_chip,
+                       pre);
         if (sp.total <= kSmemCap) break;
         if (bt == 1) return cudaErrorNotSupported;
     }
+    a.piece = piece;
+    a.c_on_chip = c_on_chip ? 1 : 0;
+    a.c_last = c_last;
     a.lbt = 0;
     while ((1 << a.lbt) < bt) ++a.lbt;
     auto aligned = [](const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; };
-    const bool ptrs = (I == 0 || aligned(a.x)) && aligned(a.h0) && aligned(a.h_seq);
+    const int xrows = pre ? 0 : I;   // staged rows that come from x_t
+    const bool ptrs = (xrows == 0 || aligned(a.x)) && aligned(a.h0) && aligned(a.h_seq);
     a.stage_mode = kStageScalar;
-    if (ptrs && a.B % 4 == 0 && bt % 4 == 0) a.stage_mode = kStageQuadCols;
-    else if (ptrs && a.B == 1 && I % 4 == 0 && H % 4 == 0) a.stage_mode = kStageQuadRows;
+    if (ptrs && B % 4 == 0 && bt % 4 == 0) a.stage_mode = kStageQuadCols;
+    else if (ptrs && B == 1 && xrows % 4 == 0 && H % 4 == 0) a.stage_mode = kStageQuadRows;
     static const cudaError_t attr = cudaFuncSetAttribute(seq_kernel<BF16, MODE>,
                                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
                                                          static_cast<int>(kSmemCap));
     if (attr != cudaSuccess) return attr;
-    // workspace: barrier word, abort flag, and the cell state unless c_last holds it
-    const size_t cbytes = kGru || c_last ? 0 : size_t(H) * size_t(a.B) * 4;
-    void *ws = nullptr;
-    cudaError_t e = cudaMallocAsync(&ws, 256 + cbytes, stream);
+    // workspace: barrier word and abort flag; the cell state when it is neither
+    // on chip nor in c_last; the x parts and the product input they come from
+    const size_t cbytes = kGru || c_on_chip || c_last ? 0 : up(size_t(H) * size_t(B) * 4);
+    const size_t ws_bytes = 256 + cbytes + (pre ? pre_bytes : 0);
+    char *ws = nullptr;
+    cudaError_t e = stream_alloc(reinterpret_cast<void **>(&ws), ws_bytes, stream);
     if (e != cudaSuccess) return e;
     e = cudaMemsetAsync(ws, 0, 16, stream);
-    a.bar = static_cast<unsigned *>(ws);
-    a.abort_flag = reinterpret_cast<int *>(static_cast<char *>(ws) + 4);
-    a.c_state = kGru ? nullptr : (c_last ? c_last : reinterpret_cast<float *>(static_cast<char *>(ws) + 256));
+    a.bar = reinterpret_cast<unsigned *>(ws);
+    a.abort_flag = reinterpret_cast<int *>(ws + 4);
+    a.c_state = kGru || c_on_chip ? nullptr : (c_last ? c_last : reinterpret_cast<float *>(ws + 256));
+    if (pre && e == cudaSuccess) {
+        float *xall = reinterpret_cast<float *>(ws + 256 + cbytes);
+        float *gx = reinterpret_cast<float *>(ws + 256 + cbytes + up(size_t(I + H) * ldx * 4));
+        e = cudaMemsetAsync(xall + size_t(I) * ldx, 0, size_t(H) * ldx * 4, stream);
+        if (e == cudaSuccess) {
+            const int64_t warps = T * I;
+            const unsigned grid = static_cast<unsigned>(std::min<int64_t>((warps + 7) / 8, int64_t(sm_count()) * 16));
+            gather_x_kernel<<<grid, 256, 0, stream>>>(a.x, a.T, I, B, xall, ldx);
+            e = cudaGetLastError();
+        }
+        if (e == cudaSuccess) e = launch_spmm(f, xall, ldx, T * B, gx, ldx, false, DARB_PATH_AUTO, stream);
+        a.gx = gx;
+        a.ldgx = ldx;
+    }
     if (e == cudaSuccess) {
         cudaLaunchConfig_t cfg = {};
         cfg.gridDim = dim3(static_cast<unsigned>(G));

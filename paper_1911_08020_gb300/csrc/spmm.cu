@@ -8,6 +8,9 @@
 // exactly once.
 #include "rowlane.cuh"
 
+#include <mutex>
+#include <set>
+
 namespace darb {
 
 cudaError_t launch_spmm(const Format &f, const float *X, int64_t ldx, int64_t batch, float *Y,
@@ -23,6 +26,29 @@ cudaError_t launch_spmm(const Format &f, const float *X, int64_t ldx, int64_t ba
                       : rowlane::launch_any<false, kModeY>(f, X, ldx, batch, Y, ldy, none, early, stream);
     }
     return launch_spmm_batch(f, X, ldx, batch, Y, ldy, early, stream);
+}
+
+cudaError_t stream_alloc(void **p, size_t bytes, cudaStream_t stream) {
+    static std::mutex mu;
+    static std::set<int> raised;
+    int dev = 0;
+    if (cudaGetDevice(&dev) == cudaSuccess) {
+        std::lock_guard<std::mutex> lk(mu);
+        if (raised.insert(dev).second) {
+            cudaMemPool_t pool;
+            uint64_t cur = 0;
+            if (cudaDeviceGetMemPool(&pool, dev) == cudaSuccess &&
+                cudaMemPoolGetAttribute(pool, cudaMemPoolAttrReleaseThreshold, &cur) == cudaSuccess &&
+                cur < kPoolKeep) {
+                uint64_t v = kPoolKeep;
+                cudaMemPoolSetAttribute(pool, cudaMemPoolAttrReleaseThreshold, &v);
+            }
+            cudaGetLastError();
+        }
+    } else {
+        cudaGetLastError();
+    }
+    return cudaMallocAsync(p, bytes, stream);
 }
 
 int sm_count() {

@@ -592,7 +592,7 @@ cudaError_t launch_kw(const Format &f, const float *X, int64_t ldx, int64_t batc
     const size_t part = (size_t(f.cols) * size_t(ldw) * 2 + 255) / 256 * 256;
     const size_t partials = ksplit > 1 ? size_t(ksplit) * T * NT * kRows * p.N * 4 : 0;
     void *ws = nullptr;
-    cudaError_t e = cudaMallocAsync(&ws, 2 * part + partials, stream);
+    cudaError_t e = stream_alloc(&ws, 2 * part + partials, stream);
     if (e != cudaSuccess) return e;
     uint16_t *hi = static_cast<uint16_t *>(ws), *lo = hi + part / 2;
     float *pt = ksplit > 1 ? reinterpret_cast<float *>(static_cast<char *>(ws) + 2 * part) : nullptr;

@@ -124,6 +124,34 @@ def test_gru_sequence_blocks_straddling_the_input_boundary():
             darb.darb_destroy(h)
 
 
+# (I, H, B, T) where x_t is at least a third of the stacked input and the
+# sequence has at least 64 columns: the x parts of all steps go through one
+# product before the recurrence; block sizes that do not divide I leave blocks
+# straddling the x/h boundary
+PRE_SHAPES = [(13, 24, 5, 13), (40, 64, 33, 2), (100, 70, 64, 3), (8, 16, 1, 64), (30, 50, 20, 4)]
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_sequences_with_precomputed_x_parts(dtype):
+    g = np.random.default_rng(45)
+    for I, H, B, T in PRE_SHAPES:
+        xs = synth.activations(T * I, B, seed=I).reshape(T, I, B)
+        h0, c0 = synth.state(H, B, seed=H), synth.state(H, B, seed=H + 1, scale=1.0)
+        stored, m = _gate_matrix(g, 4, I, H, dtype, (3, 5, 7, 8, 13))
+        h, ref = encode_both(stored, m, dtype)
+        try:
+            _check_lstm_sequence(h, ref, T, I, H, B, xs, h0, c0, synth.bias(4 * H, seed=I), TOL[dtype])
+        finally:
+            darb.darb_destroy(h)
+        stored, m = _gate_matrix(g, 3, I, H, dtype, (3, 5, 7, 8, 13))
+        h, ref = encode_both(stored, m, dtype)
+        try:
+            _check_gru_sequence(h, ref, T, I, H, B, xs, h0, synth.bias(3 * H, seed=1), synth.bias(3 * H, seed=2),
+                                TOL[dtype])
+        finally:
+            darb.darb_destroy(h)
+
+
 @pytest.mark.parametrize("name,batch", [("lstm_1024", 1), ("lstm_1024", 32), ("lstm_lm_1500", 20)])
 def test_lstm_sequence_workloads(name, batch):
     """Full-size gate matrices in the launch configuration the bench times."""
