@@ -46,6 +46,15 @@ struct SeqArgs {
     int stage_mode;         // kStage*
     int piece;              // kept weights per work item, at most
     int c_on_chip;          // LSTM: cell state in shared memory
+    // staged input rows: x_t at [0, I) (none when the x parts are precomputed),
+    // h_{t-1} from row ipad, a zero row at ipad + hpad
+    int ipad, hpad;
+    // tensor-map staging (tma != 0): boxes of {bt columns, bxh rows} over x_t
+    // (nbx of them) and {bt, bhh} over h_{t-1} (nbh), tile_bytes per tile in all;
+    // with cs = 2 the two CTAs of a cluster each load half of the boxes and
+    // multicast them to both
+    int tma, cs, nbx, bxh, nbh, bhh;
+    uint32_t tile_bytes;
     int64_t B;
     const float *gx;        // x parts of the gate sums of every step, rows x ldgx (row r, step t, column b
                             // at r * ldgx + t * B + b), or nullptr: x_t is staged with h_{t-1} instead
@@ -89,21 +98,22 @@ inline SmemPlan smem_plan(int64_t kept_cap, int rows_cap, int items_cap, int uni
     p.bias_off = take(size_t(rows_cap) * 2 * 4);
     p.c_off = take(c_on_chip ? size_t(units_cap) * size_t(B) * 4 : 0);
     p.gx_off = take(pre ? size_t(rows_cap) * bt * 4 : 0);
-    p.in_off = take(size_t(in_rows) * bt * 4);
+    p.in_off = take(size_t(in_rows) * bt * 4 + 128);   // rounded up to 128 bytes in the kernel
     p.part_off = take(size_t(gru ? 2 : 1) * items_cap * bt * 4);
     p.total = static_cast<uint32_t>(std::min<size_t>(o, UINT32_MAX));
     return p;
 }
 
-// Kept weight p of the CTA: value and absolute column.
+// Kept weight p of the CTA: its value and the index (row * bt) of the first
+// element of the staged input row it multiplies.
 template <bool BF16> struct Packed;
-template <> struct Packed<true> {   // bf16 bits << 16 | column
+template <> struct Packed<true> {   // bf16 bits << 16 | index
     using T = uint32_t;
     static __device__ __forceinline__ T make(uint32_t bits, uint32_t col) { return (bits << 16) | col; }
     static __device__ __forceinline__ float val(T w) { return __uint_as_float(w & 0xFFFF0000u); }
     static __device__ __forceinline__ uint32_t col(T w) { return w & 0xFFFFu; }
 };
-template <> struct Packed<false> {  // fp32 bits, column
+template <> struct Packed<false> {  // fp32 bits, index
     using T = uint2;
     static __device__ __forceinline__ T make(uint32_t bits, uint32_t col) { return make_uint2(bits, col); }
     static __device__ __forceinline__ float val(T w) { return __uint_as_float(w.x); }
@@ -144,25 +154,56 @@ __device__ __forceinline__ bool grid_barrier(const SeqArgs &a, unsigned target, 
     return *s_ok != 0;
 }
 
-// Sum over kept weights [pa, pb) of the CTA, subgroup `sub` taking every S-th
-// weight from pa + sub, against batch column `col` of the staged input.
-template <class P>
-__device__ __forceinline__ float dot_range(const typename P::T *s_w, const float *s_in, int pa, int pb, int sub, int S,
-                                           int lbt, int col) {
-    float acc0 = 0.0f, acc1 = 0.0f;
-    int p = pa + sub;
-    for (; p + 3 * S < pb; p += 4 * S) {
-        const typename P::T w0 = s_w[p], w1 = s_w[p + S], w2 = s_w[p + 2 * S], w3 = s_w[p + 3 * S];
-        const float v0 = s_in[(P::col(w0) << lbt) + col], v1 = s_in[(P::col(w1) << lbt) + col];
-        const float v2 = s_in[(P::col(w2) << lbt) + col], v3 = s_in[(P::col(w3) << lbt) + col];
-        acc0 = fmaf(P::val(w0), v0, acc0);
-        acc1 = fmaf(P::val(w1), v1, acc1);
-        acc0 = fmaf(P::val(w2), v2, acc0);
-        acc1 = fmaf(P::val(w3), v3, acc1);
+// On-chip layout of one row's kept weights: an x region, then an h region,
+// each padded with zero weights (pointing at the zero row of the staged input)
+// to a multiple of 4 so that a lane loads 4 weights at once.  Block jmid = I/m
+// is the only block that can hold columns on both sides of I.
+//   x parts precomputed: h region only, blocks jmid.. (an x weight of block
+//     jmid becomes a zero weight);
+//   GRU otherwise: blocks 0..jmid in the x region (block jmid there only if
+//     its weight multiplies x), blocks jmid.. in the h region;
+//   LSTM otherwise: one region of all blocks.
+__host__ __device__ inline int round4(int v) { return (v + 3) & ~3; }
+__host__ __device__ inline void row_regions(int n, int m, int I, bool pre, bool gru, int &xr, int &hr) {
+    const int jmid = I / m;
+    if (pre) {
+        xr = 0;
+        hr = round4(n - jmid);
+    } else if (gru) {
+        xr = round4(jmid + 1);
+        hr = round4(n - jmid);
+    } else {
+        xr = round4(n);
+        hr = 0;
     }
-    for (; p < pb; p += S) {
-        const typename P::T w = s_w[p];
-        acc0 = fmaf(P::val(w), s_in[(P::col(w) << lbt) + col], acc0);
+}
+
+// Sum over kept weights [pa, pb) of the CTA (multiples of 4), subgroup `sub`
+// taking every S-th group of 4 weights from pa + 4 sub, against one batch
+// column of the staged input: s_inc = s_in + that column, and a weight's
+// column field is the index of its staged row's first element, row * bt.
+template <class P>
+__device__ __forceinline__ float dot_range(const typename P::T *s_w, const float *s_inc, int pa, int pb, int sub,
+                                           int S) {
+    float acc0 = 0.0f, acc1 = 0.0f;
+#pragma unroll 2
+    for (int p = pa + 4 * sub; p < pb; p += 4 * S) {
+        typename P::T w[4];
+        if constexpr (sizeof(typename P::T) == 4) {
+            const uint4 q = *reinterpret_cast<const uint4 *>(s_w + p);
+            w[0] = q.x; w[1] = q.y; w[2] = q.z; w[3] = q.w;
+        } else {
+            const uint4 q0 = *reinterpret_cast<const uint4 *>(s_w + p);
+            const uint4 q1 = *reinterpret_cast<const uint4 *>(s_w + p + 2);
+            w[0] = make_uint2(q0.x, q0.y); w[1] = make_uint2(q0.z, q0.w);
+            w[2] = make_uint2(q1.x, q1.y); w[3] = make_uint2(q1.z, q1.w);
+        }
+        const float v0 = s_inc[P::col(w[0])], v1 = s_inc[P::col(w[1])];
+        const float v2 = s_inc[P::col(w[2])], v3 = s_inc[P::col(w[3])];
+        acc0 = fmaf(P::val(w[0]), v0, acc0);
+        acc1 = fmaf(P::val(w[1]), v1, acc1);
+        acc0 = fmaf(P::val(w[2]), v2, acc0);
+        acc1 = fmaf(P::val(w[3]), v3, acc1);
     }
     return acc0 + acc1;
 }
@@ -245,13 +286,15 @@ __device__ __forceinline__ void stage_input(const SeqArgs &a, int I, int K, cons
 
 template <bool BF16, int MODE>
 __global__ void __launch_bounds__(kThreads, 1)
-seq_kernel(Format f, SeqArgs a, Ranges rg, SmemPlan sp) {
+seq_kernel(Format f, SeqArgs a, Ranges rg, SmemPlan sp, const __grid_constant__ CUtensorMap mx,
+           const __grid_constant__ CUtensorMap mh0, const __grid_constant__ CUtensorMap mhs) {
     constexpr int kGates = MODE == kModeLstm ? 4 : 3;
     constexpr bool kGru = MODE == kModeGru;
     using P = Packed<BF16>;
     using PT = typename P::T;
     extern __shared__ __align__(16) unsigned char sm[];
-    __shared__ int s_ok, s_nitems;
+    __shared__ int s_ok, s_nitems, s_staged, s_next;
+    __shared__ __align__(8) uint64_t s_full, s_empty;   // tile landed; every CTA of the cluster done with it
     PT *s_w = reinterpret_cast<PT *>(sm + sp.w_off);
     int *s_rowptr = reinterpret_cast<int *>(sm + sp.rowptr_off);
     int *s_mid = reinterpret_cast<int *>(sm + sp.mid_off);          // GRU: first kept weight of a row on h
@@ -260,7 +303,8 @@ seq_kernel(Format f, SeqArgs a, Ranges rg, SmemPlan sp) {
     float *s_bias = reinterpret_cast<float *>(sm + sp.bias_off);    // [R] (GRU: [2R], b_ih then b_hh)
     float *s_c = reinterpret_cast<float *>(sm + sp.c_off);          // [units][B] when on chip
     float *s_gx = reinterpret_cast<float *>(sm + sp.gx_off);        // [R][bt]: x parts of this tile
-    float *s_in = reinterpret_cast<float *>(sm + sp.in_off);        // [kin + 1][bt], last row zero
+    float *s_in = reinterpret_cast<float *>(                          // [kin + 1][bt], row kin zero
+        (reinterpret_cast<uintptr_t>(sm + sp.in_off) + 127) & ~uintptr_t(127));
     float *s_part = reinterpret_cast<float *>(sm + sp.part_off);    // [parts][items][bt]
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int u0 = rg.start[blockIdx.x], nu = rg.start[blockIdx.x + 1] - u0;
@@ -272,14 +316,23 @@ seq_kernel(Format f, SeqArgs a, Ranges rg, SmemPlan sp) {
     // with the x parts precomputed only h_{t-1} is staged and only the kept
     // weights of blocks that reach column I are kept on chip (columns shifted by I)
     const bool pre = a.gx != nullptr;
-    const int kin = pre ? H : I + H, ioff = pre ? I : 0;
+    // GRU without precomputed x parts keeps the x and h sums of each item apart
+    const bool split = kGru && !pre;
+    const int kin = a.ipad + a.hpad;
+    // the cluster this CTA actually runs in: multicast and remote arrivals only
+    // when the launch really formed clusters of a.cs CTAs
+    const int cs = a.cs > 1 && cluster_nctarank() == uint32_t(a.cs) ? a.cs : 1;
+    const uint32_t rank = cs > 1 ? cluster_ctarank() : 0;
     auto grow = [&](int lr) { return (lr / nu) * H + u0 + lr % nu; };
 
     // ---- prologue: row sizes, biases, cell state, the zero row of the staged input
     for (int lr = tid; lr < R; lr += kThreads) {
         const int r = grow(lr);
         const Group &g = f.groups[f.rowloc[r] / kSlots];
-        s_rowptr[lr + 1] = g.n - (pre ? I / g.m : 0);
+        int xr, hr;
+        row_regions(g.n, g.m, I, pre, kGru, xr, hr);
+        s_rowptr[lr + 1] = xr + hr;
+        s_mid[lr] = xr;   // relative until the row pointers exist
         if constexpr (kGru) {
             s_bias[lr] = a.b_ih ? a.b_ih[r] : 0.0f;
             s_bias[R + lr] = a.b_hh ? a.b_hh[r] : 0.0f;
@@ -291,6 +344,12 @@ seq_kernel(Format f, SeqArgs a, Ranges rg, SmemPlan sp) {
         if (a.c_on_chip)
             for (int i = tid; i < nu * B; i += kThreads) s_c[i] = a.c0[int64_t(u0) * B + i];
     for (int j = tid; j < bt; j += kThreads) s_in[(kin << lbt) + j] = 0.0f;
+    if (tid == 0) {
+        mbar_init(&s_full, 1);
+        mbar_init(&s_empty, cs);
+        fence_mbar_init();
+    }
+    if (cs > 1) cluster_sync_all();   // the partner's barriers exist before anything targets them
     __syncthreads();
     // row pointers and work items: every row cut into pieces of at most a.piece weights
     if (tid == 0) {
@@ -298,6 +357,7 @@ seq_kernel(Format f, SeqArgs a, Ranges rg, SmemPlan sp) {
         for (int lr = 0; lr < R; ++lr) {
             const int n = s_rowptr[lr + 1];
             s_rowptr[lr] = p;
+            s_mid[lr] += p;
             s_rowitem[lr] = ni;
             for (int q = 0; q < n; q += a.piece) s_item[ni++] = make_int4(p + q, p + min(n, q + a.piece), lr, 0);
             p += n;
@@ -307,16 +367,16 @@ seq_kernel(Format f, SeqArgs a, Ranges rg, SmemPlan sp) {
         s_nitems = ni;
     }
     __syncthreads();
-    // every kept weight as (value, column); a row's weights are in column order
+    // zero weights everywhere, then every kept weight as (value, staged row)
+    for (int p = tid; p < s_rowptr[R]; p += kThreads) s_w[p] = P::make(0u, uint32_t(kin) << lbt);
+    __syncthreads();
     for (int lr = warp; lr < R; lr += kSeqWarps) {
         const int loc = f.rowloc[grow(lr)];
         const Group g = f.groups[loc / kSlots];
         const int slot = loc % kSlots;
-        const int base = s_rowptr[lr];
-        const int jmid = I / g.m;   // the only block that can hold columns on both sides of I
-        const int jlo = pre ? jmid : 0;
-        if (pre && lane == 0) s_mid[lr] = base;   // everything kept here multiplies h
-        for (int j = jlo + lane; j < g.n; j += 32) {
+        const int base = s_rowptr[lr], mid = s_mid[lr];
+        const int jmid = I / g.m;
+        for (int j = (pre ? jmid : 0) + lane; j < g.n; j += 32) {
             const int64_t rec = int64_t(j / kChunk) * kSlots + slot;
             const int q = j % kChunk;
             uint32_t bits;
@@ -326,29 +386,32 @@ seq_kernel(Format f, SeqArgs a, Ranges rg, SmemPlan sp) {
             if (g.nib) o = (f.offs[g.off_off + rec] >> (4 * q)) & 15u;
             else o = (f.offs[g.off_off + 2 * rec + (q >> 2)] >> (8 * (q & 3))) & 255u;
             uint32_t c = uint32_t(j) * uint32_t(g.m) + o;
-            if (pre) {
-                if (c < uint32_t(I)) {   // an x weight of the straddling block: its product is in gx
-                    bits = 0;
-                    c = uint32_t(kin);
-                } else {
-                    c -= uint32_t(ioff);
-                }
-            } else if (j == jmid) {
-                s_mid[lr] = base + j + (c < uint32_t(I) ? 1 : 0);
+            const bool on_h = c >= uint32_t(I);
+            int at;
+            if (pre || kGru) at = on_h ? mid + j - jmid : base + j;   // h region from block jmid on
+            else at = base + j;
+            if (on_h) {
+                c = c - uint32_t(I) + uint32_t(a.ipad);   // staged row of h
+            } else if (pre) {   // an x weight of block jmid: its product is in gx
+                bits = 0;
+                c = uint32_t(kin);
+                at = mid;
             }
-            s_w[base + j - jlo] = P::make(bits, c);
+            s_w[at] = P::make(bits, c << lbt);   // (kin + 1) * bt floats fit in shared memory: < 2^16
         }
     }
     __syncthreads();
     const int NI = s_nitems;
+    if (tid == 0) s_next = 0;
     for (int i = tid; i < NI; i += kThreads) {
         int4 it = s_item[i];
-        it.w = kGru ? max(it.x, min(it.y, s_mid[it.z])) : it.y;
+        it.w = split ? max(it.x, min(it.y, s_mid[it.z])) : it.y;
         s_item[i] = it;
     }
     __syncthreads();
 
     // ---- the steps
+    int tile = 0;   // tiles staged so far: the parity of both barriers
     float *c_run = kGru ? nullptr : (a.c_on_chip ? s_c : a.c_state + int64_t(u0) * B);
     for (int t = 0; t < a.T; ++t) {
         const float *xt = a.x + int64_t(t) * I * B;
@@ -359,34 +422,66 @@ seq_kernel(Format f, SeqArgs a, Ranges rg, SmemPlan sp) {
         for (int64_t b0 = 0; b0 < B; b0 += bt) {
             const int nb = static_cast<int>(B - b0 < bt ? B - b0 : bt);
             // stage [x_t; h_{t-1}] (or h_{t-1}) for columns [b0, b0 + nb), zeros past the batch
+            if (a.tma && tid == 0) {
+                // every CTA of the cluster is done with the previous tile
+                bool ok = tile == 0 || mbar_wait_cluster(&s_empty, (tile - 1) & 1);
+                if (ok) {
+                    fence_proxy_async_global();   // h_{t-1} was published by generic stores
+                    mbar_arrive_expect_tx(&s_full, a.tile_bytes);
+                    for (int bx = static_cast<int>(rank); bx < a.nbx + a.nbh; bx += cs) {
+                        const bool isx = bx < a.nbx;
+                        const int y = isx ? bx * a.bxh : (bx - a.nbx) * a.bhh;
+                        float *dst = s_in + (int64_t(isx ? y : a.ipad + y) << lbt);
+                        const CUtensorMap *m = isx ? &mx : (t == 0 ? &mh0 : &mhs);
+                        const int z = isx ? t : (t == 0 ? 0 : t - 1);
+                        if (cs > 1) tensor3d_g2s_multicast(dst, m, static_cast<int>(b0), y, z, &s_full, 3);
+                        else tensor3d_g2s(dst, m, static_cast<int>(b0), y, z, &s_full);
+                    }
+                    ok = mbar_wait(&s_full, tile & 1, false);
+                }
+                if (!ok) {
+                    atomicOr(a.status, kStatusTimeout);
+                    atomicExch(a.abort_flag, 1);
+                }
+                s_staged = ok;
+            }
             if (pre)
                 for (int i = tid; i < R << lbt; i += kThreads) {
                     const int lr = i >> lbt, j = i & (bt - 1);
                     s_gx[i] = j < nb ? __ldg(a.gx + int64_t(grow(lr)) * a.ldgx + int64_t(t) * B + b0 + j) : 0.0f;
                 }
-            stage_input(a, pre ? 0 : I, kin, xt, hp, b0, nb, s_in);
+            if (!a.tma) stage_input(a, pre ? 0 : I, kin, xt, hp, b0, nb, s_in);
             __syncthreads();
-            // partial gate sums of the work items; items go to warps in a snake
-            for (int r0 = 0; r0 < NI; r0 += kSeqWarps) {
-                const int ii = r0 + (((r0 / kSeqWarps) & 1) ? kSeqWarps - 1 - warp : warp);
-                if (ii >= NI) continue;
+            if (a.tma) {
+                if (!s_staged) return;
+                mbar_wait(&s_full, tile & 1, false);   // completed: makes the copied data visible to this thread
+            }
+            // partial gate sums of the work items, handed out to warps as they come free
+            while (true) {
+                int ii = 0;
+                if (lane == 0) ii = atomicAdd(&s_next, 1);
+                ii = __shfl_sync(0xFFFFFFFFu, ii, 0);
+                if (ii >= NI) break;
                 const int4 it = s_item[ii];
-                float ax = dot_range<P>(s_w, s_in, it.x, it.w, sub, S, lbt, col);
-                float ah = 0.0f;
-                if constexpr (kGru) ah = dot_range<P>(s_w, s_in, it.w, it.y, sub, S, lbt, col);
+                float a0 = dot_range<P>(s_w, s_in + col, it.x, it.w, sub, S);
+                float a1 = 0.0f;
+                if (split) a1 = dot_range<P>(s_w, s_in + col, it.w, it.y, sub, S);
                 for (int o = 16; o >= bt; o >>= 1) {
-                    ax += __shfl_xor_sync(0xFFFFFFFFu, ax, o);
-                    if constexpr (kGru) ah += __shfl_xor_sync(0xFFFFFFFFu, ah, o);
+                    a0 += __shfl_xor_sync(0xFFFFFFFFu, a0, o);
+                    if (split) a1 += __shfl_xor_sync(0xFFFFFFFFu, a1, o);
                 }
                 if (sub == 0) {
-                    s_part[(ii << lbt) + col] = ax;
-                    if constexpr (kGru) s_part[((NI + ii) << lbt) + col] = ah;
+                    s_part[(ii << lbt) + col] = a0;
+                    if (split) s_part[((NI + ii) << lbt) + col] = a1;
                 }
             }
             __syncthreads();
+            if (tid == 0) s_next = 0;   // for the next tile; every warp has left the loop
             // the cells of the owned units for these columns
-            auto gate = [&](int lr, int part, int j) {
-                float v = s_bias[part * R + lr];
+            // partial sums of local row lr: part 0 (everything, or the x part of a
+            // split GRU row), part 1 (the h part of a split GRU row)
+            auto sum = [&](int lr, int part, int j) {
+                float v = 0.0f;
                 for (int ii = s_rowitem[lr]; ii < s_rowitem[lr + 1]; ++ii) v += s_part[((part * NI + ii) << lbt) + j];
                 return v;
             };
@@ -396,24 +491,32 @@ seq_kernel(Format f, SeqArgs a, Ranges rg, SmemPlan sp) {
                 const int64_t e = int64_t(ui) * B + b0 + j;
                 auto xg = [&](int lr) { return pre ? s_gx[(lr << lbt) + j] : 0.0f; };
                 if constexpr (MODE == kModeLstm) {
-                    const float pi = gate(ui, 0, j) + xg(ui), pf = gate(nu + ui, 0, j) + xg(nu + ui);
-                    const float pg = gate(2 * nu + ui, 0, j) + xg(2 * nu + ui);
-                    const float po = gate(3 * nu + ui, 0, j) + xg(3 * nu + ui);
+                    auto gate = [&](int lr) { return s_bias[lr] + sum(lr, 0, j) + xg(lr); };
+                    const float pi = gate(ui), pf = gate(nu + ui), pg = gate(2 * nu + ui), po = gate(3 * nu + ui);
                     const float c = sigm(pf) * cp[e] + sigm(pi) * tanhf(pg);
                     c_run[e] = c;
                     if (ct) ct[e] = c;
                     ht[e] = sigm(po) * tanhf(c);
                 } else {
-                    const float rr = sigm(gate(ui, 0, j) + xg(ui) + gate(ui, 1, j));
-                    const float zz = sigm(gate(nu + ui, 0, j) + xg(nu + ui) + gate(nu + ui, 1, j));
-                    const float nn = tanhf(gate(2 * nu + ui, 0, j) + xg(2 * nu + ui) + rr * gate(2 * nu + ui, 1, j));
-                    ht[e] = (1.0f - zz) * nn + zz * s_in[((kin - H + u0 + ui) << lbt) + j];
+                    // x part (b_ih + W_x x) and h part (b_hh + W_h h) of each gate
+                    auto gx_ = [&](int lr) { return s_bias[lr] + (pre ? xg(lr) : sum(lr, 0, j)); };
+                    auto gh_ = [&](int lr) { return s_bias[R + lr] + sum(lr, split ? 1 : 0, j); };
+                    const float rr = sigm(gx_(ui) + gh_(ui));
+                    const float zz = sigm(gx_(nu + ui) + gh_(nu + ui));
+                    const float nn = tanhf(gx_(2 * nu + ui) + rr * gh_(2 * nu + ui));
+                    ht[e] = (1.0f - zz) * nn + zz * s_in[((a.ipad + u0 + ui) << lbt) + j];
                 }
             }
             __syncthreads();
+            if (a.tma && tid == 0)   // this CTA is done with the tile: tell every CTA of the cluster
+                for (int r = 0; r < cs; ++r) mbar_arrive_cluster(&s_empty, static_cast<uint32_t>(r));
+            ++tile;
         }
         if (t + 1 < a.T && !grid_barrier(a, unsigned(t + 1) * gridDim.x, &s_ok)) return;
     }
+    // the partner's last arrival on this CTA's barrier has landed before it leaves
+    if (a.tma && cs > 1 && tid == 0 && !mbar_wait_cluster(&s_empty, (tile - 1) & 1))
+        atomicOr(a.status, kStatusTimeout);
     if constexpr (!kGru)
         if (a.c_on_chip && a.c_last)
             for (int i = tid; i < nu * B; i += kThreads) a.c_last[int64_t(u0) * B + i] = s_c[i];
@@ -484,8 +587,10 @@ static cudaError_t launch_seq_t(const Format &f, const int32_t *row_m, seq::SeqA
     const bool pre = precompute_x(T, I, H, B, pre_bytes);
     // kept weights on chip per row: all, or those of the blocks that reach column I
     auto row_kept = [&](int64_t r) {
-        const int64_t m = row_m[r];
-        return (f.cols + m - 1) / m - (pre ? I / m : 0);
+        const int m = row_m[r];
+        int xr, hr;
+        row_regions(static_cast<int>((f.cols + m - 1) / m), m, I, pre, kGru, xr, hr);
+        return int64_t(xr + hr);
     };
     std::vector<int64_t> kept(static_cast<size_t>(H));
     for (int u = 0; u < H; ++u) {
@@ -493,45 +598,80 @@ static cudaError_t launch_seq_t(const Format &f, const int32_t *row_m, seq::SeqA
         for (int q = 0; q < kGates; ++q) k += row_kept(int64_t(q) * H + u);
         kept[static_cast<size_t>(u)] = k;
     }
-    const int G = std::max(1, std::min({sm_count(), H, kMaxCtas}));
+    auto aligned = [](const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; };
+    const int xrows = pre ? 0 : I;   // staged rows that come from x_t
+    const bool ptrs = (xrows == 0 || aligned(a.x)) && aligned(a.h0) && aligned(a.h_seq);
+    // tensor-map staging needs 16-byte rows of every source (B a multiple of 4)
+    const bool tma_ok = ptrs && B % 4 == 0 && tensor_map_encoder() != nullptr;
+    int G = std::max(1, std::min({sm_count(), H, kMaxCtas}));
+    if (tma_ok && G >= 2) G &= ~1;   // clusters of two CTAs share each staged tile
     Ranges rg{};
     int64_t kept_cap = 0;
     int units_cap = 0;
     split_units(kept, G, rg, kept_cap, units_cap);
     if (kept_cap > (int64_t(1) << 20)) return cudaErrorNotSupported;
     const bool c_on_chip = !kGru && size_t(units_cap) * size_t(B) * 4 <= kCellOnChip;
-    const int kin = pre ? H : I + H;
-    // widest batch tile (a power of two, <= 32) whose staging still fits; rows
-    // are cut into work items of about kept_cap / (2 * warps) weights, and of at
-    // least 8 weights per lane of a subgroup
+    // staged rows per box: at most 256, and a multiple of 32 / bt so that every
+    // box lands on a 128-byte boundary; as few padding rows as possible
+    auto box_rows = [](int n, int align, int &nbox, int &rows) {
+        nbox = (n + 255) / 256;
+        rows = nbox ? ((n + nbox - 1) / nbox + align - 1) / align * align : 0;
+        if (rows > 256) rows = 256 / align * align, nbox = (n + rows - 1) / rows;
+    };
+    int nbx = 0, bxh = 0, nbh = 0, bhh = 0;
+    // widest batch tile (a power of two, <= 32) whose staging still fits, with
+    // rows cut into work items of about kept_cap / (ipw * warps) weights (a
+    // multiple of 4, at least 2 loads of 4 weights per subgroup): ipw = 4 items
+    // per warp balances the warps best, fewer save the items' partial sums
     int bt = 1;
     while (bt < kMaxTile && bt < B) bt *= 2;
     SmemPlan sp{};
     int piece = 0;
-    for (;; bt /= 2) {
+    for (bool fits = false; !fits; bt /= 2) {
+        if (bt == 0) return cudaErrorNotSupported;
         const int S = kMaxTile / bt;
-        piece = static_cast<int>(std::max<int64_t>(8 * S, (kept_cap + 2 * kSeqWarps - 1) / (2 * kSeqWarps)));
-        int items_cap = 0;
-        for (int q = 0; q < G; ++q) {
-            int items = 0;
-            for (int g = 0; g < kGates; ++g)
-                for (int u = rg.start[q]; u < rg.start[q + 1]; ++u)
-                    items += static_cast<int>((row_kept(int64_t(g) * H + u) + piece - 1) / piece);
-            items_cap = std::max(items_cap, items);
+        const bool tma = tma_ok && bt >= 4;
+        if (tma) {
+            box_rows(xrows, 32 / bt, nbx, bxh);
+            box_rows(H, 32 / bt, nbh, bhh);
         }
-        sp = smem_plan(kept_cap, kGates * units_cap, items_cap, units_cap, BF16, kGru, kin + 1, bt, B, c_on_chip,
-                       pre);
-        if (sp.total <= kSmemCap) break;
-        if (bt == 1) return cudaErrorNotSupported;
+        const int in_rows = tma ? nbx * bxh + nbh * bhh + 1 : xrows + H + 1;
+        for (int ipw = 4; ipw >= 1 && !fits; ipw /= 2) {
+            piece = round4(static_cast<int>(
+                std::max<int64_t>(8 * S, (kept_cap + ipw * kSeqWarps - 1) / (ipw * kSeqWarps))));
+            int items_cap = 0;
+            for (int q = 0; q < G; ++q) {
+                int items = 0;
+                for (int g = 0; g < kGates; ++g)
+                    for (int u = rg.start[q]; u < rg.start[q + 1]; ++u)
+                        items += static_cast<int>((row_kept(int64_t(g) * H + u) + piece - 1) / piece);
+                items_cap = std::max(items_cap, items);
+            }
+            sp = smem_plan(kept_cap, kGates * units_cap, items_cap, units_cap, BF16, kGru && !pre, in_rows, bt, B,
+                           c_on_chip, pre);
+            fits = sp.total <= kSmemCap;
+        }
+        if (fits) break;
     }
     a.piece = piece;
     a.c_on_chip = c_on_chip ? 1 : 0;
     a.c_last = c_last;
     a.lbt = 0;
     while ((1 << a.lbt) < bt) ++a.lbt;
-    auto aligned = [](const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; };
-    const int xrows = pre ? 0 : I;   // staged rows that come from x_t
-    const bool ptrs = (xrows == 0 || aligned(a.x)) && aligned(a.h0) && aligned(a.h_seq);
+    a.tma = tma_ok && bt >= 4 ? 1 : 0;
+    a.cs = a.tma && G % 2 == 0 ? 2 : 1;
+    if (a.tma) {
+        a.nbx = nbx;
+        a.bxh = bxh;
+        a.nbh = nbh;
+        a.bhh = bhh;
+        a.ipad = nbx * bxh;
+        a.hpad = nbh * bhh;
+        a.tile_bytes = static_cast<uint32_t>((a.ipad + a.hpad) * bt * 4);
+    } else {
+        a.ipad = xrows;
+        a.hpad = H;
+    }
     a.stage_mode = kStageScalar;
     if (ptrs && B % 4 == 0 && bt % 4 == 0) a.stage_mode = kStageQuadCols;
     else if (ptrs && B == 1 && xrows % 4 == 0 && H % 4 == 0) a.stage_mode = kStageQuadRows;
@@ -539,6 +679,54 @@ static cudaError_t launch_seq_t(const Format &f, const int32_t *row_m, seq::SeqA
                                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
                                                          static_cast<int>(kSmemCap));
     if (attr != cudaSuccess) return attr;
+    // tensor maps of the staged sources: 3-D (batch, rows, step) so that a box
+    // running past the last row of a step reads zeros, never the next step
+    CUtensorMap mx{}, mh0{}, mhs{};
+    if (a.tma) {
+        auto make = [&](CUtensorMap *m, const float *base, int64_t rows, int64_t depth, int boxh) {
+            const cuuint64_t dims[3] = {cuuint64_t(B), cuuint64_t(rows), cuuint64_t(depth)};
+            const cuuint64_t strides[2] = {cuuint64_t(B) * 4, cuuint64_t(B) * 4 * cuuint64_t(rows)};
+            const cuuint32_t box[3] = {cuuint32_t(bt), cuuint32_t(boxh), 1};
+            const cuuint32_t es[3] = {1, 1, 1};
+            return tensor_map_encoder()(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3, const_cast<float *>(base), dims,
+                                        strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+                                        CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+        };
+        bool ok = make(&mh0, a.h0, H, 1, bhh) && make(&mhs, a.h_seq, H, T, bhh);
+        if (ok && nbx) ok = make(&mx, a.x, I, T, bxh);
+        if (!ok) {   // plain loads instead (the plan above has room for either)
+            a.tma = 0;
+            a.cs = 1;
+            a.ipad = xrows;
+            a.hpad = H;
+        }
+    }
+    cudaLaunchAttribute at[2];
+    at[0].id = cudaLaunchAttributeCooperative;
+    at[0].val.cooperative = 1;
+    at[1].id = cudaLaunchAttributeClusterDimension;
+    at[1].val.clusterDim.x = 2;
+    at[1].val.clusterDim.y = 1;
+    at[1].val.clusterDim.z = 1;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(static_cast<unsigned>(G));
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = sp.total;
+    cfg.stream = stream;
+    cfg.attrs = at;
+    cfg.numAttrs = 1;
+    if (a.cs == 2) {   // clusters of two, if that many pairs fit at once
+        cfg.numAttrs = 2;
+        cfg.attrs = at + 1;
+        int pairs = 0;
+        if (cudaOccupancyMaxActiveClusters(&pairs, seq_kernel<BF16, MODE>, &cfg) != cudaSuccess || 2 * pairs < G) {
+            cudaGetLastError();
+            a.cs = 1;
+        }
+        cfg.attrs = at;
+        cfg.numAttrs = a.cs == 2 ? 2 : 1;
+    }
     // workspace: barrier word and abort flag; the cell state when it is neither
     // on chip nor in c_last; the x parts and the product input they come from
     const size_t cbytes = kGru || c_on_chip || c_last ? 0 : up(size_t(H) * size_t(B) * 4);
@@ -564,19 +752,7 @@ static cudaError_t launch_seq_t(const Format &f, const int32_t *row_m, seq::SeqA
         a.gx = gx;
         a.ldgx = ldx;
     }
-    if (e == cudaSuccess) {
-        cudaLaunchConfig_t cfg = {};
-        cfg.gridDim = dim3(static_cast<unsigned>(G));
-        cfg.blockDim = dim3(kThreads);
-        cfg.dynamicSmemBytes = sp.total;
-        cfg.stream = stream;
-        cudaLaunchAttribute at[1];
-        at[0].id = cudaLaunchAttributeCooperative;
-        at[0].val.cooperative = 1;
-        cfg.attrs = at;
-        cfg.numAttrs = 1;
-        e = cudaLaunchKernelEx(&cfg, seq_kernel<BF16, MODE>, f, a, rg, sp);
-    }
+    if (e == cudaSuccess) e = cudaLaunchKernelEx(&cfg, seq_kernel<BF16, MODE>, f, a, rg, sp, mx, mh0, mhs);
     const cudaError_t ef = cudaFreeAsync(ws, stream);
     return e != cudaSuccess ? e : ef;
 }

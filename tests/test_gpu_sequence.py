@@ -70,9 +70,10 @@ def _check_gru_sequence(h, ref, T, I, H, B, xs, h0, bi, bh, tol):
 
 
 # (I, H, B): one unit per CTA, ragged batch tiles, several tiles, I = 0, more
-# units than CTAs, a batch tile of one column
+# units than CTAs, a batch tile of one column; batches that are multiples of 4
+# stage through tensor maps (one CTA, clusters of two, a ragged second tile)
 SHAPES = [(0, 5, 1), (3, 4, 2), (7, 33, 3), (20, 40, 8), (64, 100, 9), (10, 70, 33), (16, 300, 1),
-          (40, 200, 70), (5, 400, 17)]
+          (40, 200, 70), (5, 400, 17), (4, 1, 8), (6, 9, 4), (12, 36, 40), (0, 64, 12), (300, 260, 4)]
 
 
 @pytest.mark.parametrize("dtype", ["f32", "bf16"])
