@@ -133,9 +133,11 @@ __device__ __forceinline__ void split2(float a, float b, uint32_t *hi, uint32_t 
 // hi, lo: cols x batch bf16 with row pitch ldw (a multiple of 8).  Each thread
 // takes four consecutive batch columns of one row.
 __global__ void __launch_bounds__(256)
-split_kernel(const float *X, int64_t ldx, int64_t batch, int64_t cols, uint16_t *hi, uint16_t *lo, int64_t ldw) {
+split_kernel(const float *X, int64_t ldx, int64_t batch, int64_t cols, uint16_t *hi, uint16_t *lo, int64_t ldw,
+             int *arrive, int narrive) {
     pdl_launch_dependents();
     pdl_wait_previous();   // X may come from the previous kernel; the workspace may still be read by it
+    for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < narrive; i += gridDim.x * blockDim.x) arrive[i] = 0;
     const int64_t q4 = (batch + 3) / 4;
     const bool vec = (ldx & 3) == 0 && (reinterpret_cast<uintptr_t>(X) & 15) == 0;
     for (int64_t i = int64_t(blockIdx.x) * blockDim.x + threadIdx.x; i < cols * q4;
@@ -163,7 +165,7 @@ split_kernel(const float *X, int64_t ldx, int64_t batch, int64_t cols, uint16_t 
 template <int KW>
 __global__ void __launch_bounds__(kThreads, 1)
 tc_kernel(const __grid_constant__ CUtensorMap hmap, const __grid_constant__ CUtensorMap lmap, Format f, int ksplit,
-          int nstages, int N, int64_t batch, float *Y, int64_t ldy, float *part, int early) {
+          int nstages, int N, int64_t batch, float *Y, int64_t ldy, float *part, int *arrive, int early) {
     using G = Geo<KW>;
     constexpr int kK = KW;
     constexpr int kARow = G::kARow, kAHalf = G::kAHalf;
@@ -459,7 +461,38 @@ tc_kernel(const __grid_constant__ CUtensorMap hmap, const __grid_constant__ CUte
                 __syncwarp();
             }
         }
-        cg::this_cluster().sync();   // release/acquire: every rank's partial tile is visible
+        if (arrive == nullptr) {
+            cg::this_cluster().sync();   // release/acquire: every rank's partial tile is visible
+        } else {
+            // the ranks of the tile are CTAs of a cooperative launch: count in, then
+            // wait (bounded) until every rank has published its partial tile
+            __shared__ int s_go;
+            __syncthreads();
+            if (tid == 0) {
+                int *ctr = arrive + blockIdx.y * (gridDim.x / ksplit) + tile;
+                __threadfence();
+                atomicAdd(ctr, 1);
+                const unsigned long long t0 = global_timer_ns();
+                int go = 1;
+                while (true) {
+                    int v;
+                    asm volatile("ld.acquire.gpu.global.s32 %0, [%1];" : "=r"(v) : "l"(ctr) : "memory");
+                    if (v >= ksplit) break;
+                    if (global_timer_ns() - t0 > kWaitLimitNs) {
+                        go = 0;
+                        break;
+                    }
+                    __nanosleep(32);
+                }
+                __threadfence();
+                s_go = go;
+            }
+            __syncthreads();
+            if (!s_go) {
+                if (tid == 0) atomicOr(f.status, kStatusTimeout);
+                goto finish;
+            }
+        }
         const float *first = mine - size_t(rank) * kRows * N;   // rank 0's tile
         const int own = (kRows + ksplit - 1) / ksplit;       // rows each rank adds up
         const int r0 = rank * own, r1 = min(kRows, r0 + own);
@@ -497,6 +530,7 @@ tc_kernel(const __grid_constant__ CUtensorMap hmap, const __grid_constant__ CUte
         }
     }
 
+finish:
     if (!ok) atomicOr(f.status, kStatusTimeout);
     tc_fence_before_sync();
     __syncthreads();
@@ -553,6 +587,22 @@ inline int active_clusters(int ksplit, const Plan &p) {
     return n;
 }
 
+// CTAs of this kernel that fit on the device at once (for a cooperative launch).
+template <int KW>
+inline int64_t coop_capacity(const Plan &p) {
+    static int cache[4] = {};
+    const int wi = p.N == 32 ? 0 : p.N == 64 ? 1 : p.N == 128 ? 2 : 3;
+    if (cache[wi] == 0) {
+        int per_sm = 0;
+        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, tc_kernel<KW>, kThreads, p.smem) != cudaSuccess) {
+            cudaGetLastError();
+            per_sm = 0;
+        }
+        cache[wi] = per_sm > 0 ? per_sm * sm_count() : -1;
+    }
+    return cache[wi] > 0 ? cache[wi] : 0;
+}
+
 // Cluster split: fewest waves per unit of work, i.e. the smallest
 // ceil(units / resident clusters) / ksplit, never more ranks than stages.
 template <int KW>
@@ -586,16 +636,26 @@ cudaError_t launch_kw(const Format &f, const float *X, int64_t ldx, int64_t batc
     const int T = (f.ngroups + kCtaGroups - 1) / kCtaGroups;
     const int64_t NT = (batch + p.N - 1) / p.N;
     const int KS = static_cast<int>((f.cols + KW - 1) / KW);
-    const int ksplit = pick_split<KW>(int64_t(T) * NT, KS, p);
-    // workspace: hi and lo parts of X, then the partial tiles of a split
+    const int64_t units = int64_t(T) * NT;
+    int ksplit = pick_split<KW>(units, KS, p);
+    // A cooperative launch (every CTA resident at once) lets the ranks of a tile
+    // meet on a counter instead of a cluster barrier, so the split is not held
+    // to the cluster shapes a GPC can place: up to 8 ranks as long as one wave
+    // of CTAs holds every tile.
+    const int coop_split = static_cast<int>(std::min<int64_t>({8, int64_t(KS), coop_capacity<KW>(p) / units}));
+    const bool coop = coop_split > ksplit;
+    const int kmax = coop ? coop_split : ksplit;
+    // workspace: hi and lo parts of X, the partial tiles of a split, the tiles' arrival counters
     const int64_t ldw = (batch + 7) / 8 * 8;
     const size_t part = (size_t(f.cols) * size_t(ldw) * 2 + 255) / 256 * 256;
-    const size_t partials = ksplit > 1 ? size_t(ksplit) * T * NT * kRows * p.N * 4 : 0;
+    const size_t partials = kmax > 1 ? size_t(kmax) * units * kRows * p.N * 4 : 0;
+    const size_t counters = coop ? size_t(units) * 4 : 0;
     void *ws = nullptr;
-    cudaError_t e = stream_alloc(&ws, 2 * part + partials, stream);
+    cudaError_t e = stream_alloc(&ws, 2 * part + partials + counters, stream);
     if (e != cudaSuccess) return e;
     uint16_t *hi = static_cast<uint16_t *>(ws), *lo = hi + part / 2;
-    float *pt = ksplit > 1 ? reinterpret_cast<float *>(static_cast<char *>(ws) + 2 * part) : nullptr;
+    float *pt = kmax > 1 ? reinterpret_cast<float *>(static_cast<char *>(ws) + 2 * part) : nullptr;
+    int *arrive = coop ? reinterpret_cast<int *>(static_cast<char *>(ws) + 2 * part + partials) : nullptr;
     CUtensorMap hmap, lmap;
     std::memset(&hmap, 0, sizeof(hmap));
     std::memset(&lmap, 0, sizeof(lmap));
@@ -605,11 +665,36 @@ cudaError_t launch_kw(const Format &f, const float *X, int64_t ldx, int64_t batc
     }
     const int64_t items = f.cols * ((batch + 3) / 4);
     const unsigned sgrid = static_cast<unsigned>(std::min<int64_t>((items + 255) / 256, int64_t(sm_count()) * 8));
-    e = launch_ex(split_kernel, dim3(sgrid), dim3(256), 0, stream, 1, true, X, ldx, batch, f.cols, hi, lo, ldw);
-    if (e == cudaSuccess) {
+    e = launch_ex(split_kernel, dim3(sgrid), dim3(256), 0, stream, 1, true, X, ldx, batch, f.cols, hi, lo, ldw,
+                  arrive, static_cast<int>(counters / 4));
+    if (e == cudaSuccess && coop) {
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3(static_cast<unsigned>(T * coop_split), static_cast<unsigned>(NT));
+        cfg.blockDim = dim3(kThreads);
+        cfg.dynamicSmemBytes = p.smem;
+        cfg.stream = stream;
+        cudaLaunchAttribute attr[2];
+        attr[0].id = cudaLaunchAttributeCooperative;
+        attr[0].val.cooperative = 1;
+        attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        attr[1].val.programmaticStreamSerializationAllowed = 1;
+        cfg.attrs = attr;
+        cfg.numAttrs = 2;
+        e = cudaLaunchKernelEx(&cfg, tc_kernel<KW>, hmap, lmap, f, coop_split, p.nstages, p.N, batch, Y, ldy, pt,
+                               arrive, early ? 1 : 0);
+        if (e != cudaSuccess) {   // not launchable cooperatively here: the cluster split instead
+            cudaGetLastError();
+            e = cudaSuccess;
+            arrive = nullptr;
+        } else {
+            ksplit = 0;   // launched
+        }
+    }
+    if (e == cudaSuccess && ksplit > 0) {
         const dim3 grid(static_cast<unsigned>(T * ksplit), static_cast<unsigned>(NT));
         e = launch_ex(tc_kernel<KW>, grid, dim3(kThreads), p.smem, stream, static_cast<unsigned>(ksplit), true, hmap,
-                      lmap, f, ksplit, p.nstages, p.N, batch, Y, ldy, pt, early ? 1 : 0);
+                      lmap, f, ksplit, p.nstages, p.N, batch, Y, ldy, pt, static_cast<int *>(nullptr),
+                      early ? 1 : 0);
     }
     const cudaError_t ef = cudaFreeAsync(ws, stream);
     return e != cudaSuccess ? e : ef;
