@@ -46,6 +46,7 @@ def parse_args():
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu", action="store_true")
     p.add_argument("--no-rnn", action="store_true")
+    p.add_argument("--no-baselines", action="store_true", help="skip the cuSPARSE comparison section")
     p.add_argument("--cpu-seconds", type=float, default=30.0,
                    help="CPU time budget of the oracle arm (--impl reference) over all its steps")
     p.add_argument("--calls", default="",
@@ -445,6 +446,8 @@ def run_gpu(args, world, rank, local):
     if not args.no_rnn and not only:
         result["rnn"] = run_rnn(torch, darb, synth, peak)
         result["assign"] = run_assign(torch, darb, wl, peak)
+    if not args.no_baselines and not only:
+        result["baselines"] = run_baselines(torch, darb, wl)
     if not args.no_e2e:
         result["e2e"] = run_e2e(args, wl, torch, darb)
     wl.close()
@@ -477,6 +480,72 @@ def run_assign(torch, darb, wl, peak, reps=3):
                                             "hbm_frac": round(nbytes / (best * 1e-3) / 1e9 / peak, 4),
                                             "note": "three reads of W (two radix passes and the row count)"
                                                     " plus the host rounding rule and the copies"}
+    return out
+
+
+def run_baselines(torch, darb, wl, reps=20):
+    """darb_spmm next to cuSPARSE on the formats the paper compares with
+    (Sec. 4.2): the same kept weights as CSR, and 4x4 / 8x8 block pruning of
+    the same W at the same density as BSR (fp32 values, fp32 X and Y for the
+    vendor library).  Each product is timed alone: `reps` calls captured in a
+    CUDA graph and replayed, CUDA events around the replay; the matrices stay
+    L2-resident across the calls for every format alike."""
+    from paper_1911_08020_gb300 import baselines
+    dev = wl.dev
+
+    def timed(fn):
+        fn()
+        torch.cuda.synchronize()
+        try:
+            g = capture(torch, lambda: [fn() for _ in range(reps)])
+            run = g.replay
+        except RuntimeError:   # not capturable: launched eagerly instead
+            run = lambda: [fn() for _ in range(reps)]
+        run()
+        torch.cuda.synchronize()
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record()
+        run()
+        b.record()
+        torch.cuda.synchronize()
+        return a.elapsed_time(b) * 1e3 / reps   # us per call
+
+    out = {}
+    for mi, mat in enumerate(wl.mats):
+        name = "fc6" if mi == 0 else "fc7"
+        rows, cols, nnzb = mat["rows"], mat["cols"], mat["info"]["nnzb"]
+        rp, ci, vv = baselines.csr_from_darb(mat["h"])
+        csr = [torch.from_numpy(a).to(dev) for a in (rp, ci, vv)]
+        Wf = (mat["bits"].astype(np.uint32) << 16).view(np.float32)
+        bsr = {}
+        for bs in (4, 8):
+            brp, bci, bvals, _ = baselines.block_prune(Wf, bs, round(nnzb / (bs * bs)))
+            bsr[bs] = [torch.from_numpy(a).to(dev) for a in (brp, bci, bvals.reshape(-1))]
+        entry = {"rows": rows, "cols": cols, "kept_weights": {"darb": nnzb, "csr": int(len(vv)),
+                 "bsr4": int(bsr[4][1].numel() * 16), "bsr8": int(bsr[8][1].numel() * 64)}}
+        for B in BATCHES:
+            X = torch.randn((cols, B), device=dev)
+            Y = torch.empty((rows, B), device=dev)
+            XT = X.t().contiguous()                       # the same X, each batch column contiguous
+            YT = torch.empty((B, rows), device=dev)
+            t_darb = timed(lambda: darb.darb_spmm(mat["h"], X, Y))
+            row = {"darb_us": round(t_darb, 2)}
+            # each vendor product in the dense layout it runs fastest in (the layout change is not timed)
+            for fmt, call in [("csr", lambda Xd, Yd, lay: baselines.csr_spmm(*csr, rows, cols, Xd, Yd, lay))] + \
+                             [(f"bsr{bs}", (lambda bs_: lambda Xd, Yd, lay: baselines.bsr_spmm(
+                                 *bsr[bs_], rows, cols, bs_, Xd, Yd, lay))(bs)) for bs in (4, 8)]:
+                t_rows = timed(lambda: call(X, Y, baselines.DENSE_ROWS))
+                t_cols = timed(lambda: call(XT, YT, baselines.DENSE_COLS))
+                row[f"{fmt}_us"] = round(min(t_rows, t_cols), 2)
+                row[f"{fmt}_layout"] = "rows" if t_rows <= t_cols else "cols"
+            row["darb_speedup_vs"] = {f: round(row[f"{f}_us"] / t_darb, 2) for f in ("csr", "bsr4", "bsr8")}
+            entry[f"b{B}"] = row
+        out[name] = entry
+    out["note"] = ("cuSPARSE SpMM, fp32 values and compute, in the faster of the two dense layouts (batch "
+                   "contiguous, or each batch column contiguous; the transposition is not timed); CSR = DARB's "
+                   "kept weights; BSR = the largest-L1 bs x bs blocks of the same W at the same kept-weight "
+                   "count; darb_spmm with bf16 values as in the step; every matrix L2-resident")
     return out
 
 

@@ -87,7 +87,7 @@ DARB_API darb_status_t darb_assign_block_sizes(const int64_t *row_nnz, int64_t r
 
 /*
  * Block sizes from the weights themselves (Sec. 3.2): the K = `keep` weights
- * of largest magnitude form the mask of irregular pruning (Sec. 2.2), used
+ * of largest magnitude form the mask of irregular pruning (Sec. 2, "Irregular Pruning"), used
  * only to measure each row's density; darb_assign_block_sizes then turns the
  * row counts into block sizes.  Weights tied with the K-th largest magnitude
  * all count (the paper does not break such ties), so the counts may add up to

@@ -8,7 +8,7 @@
  * Every function is the plain definition of one step of the method, written as
  * loops in the paper's order, accumulating in double precision:
  *
- *   oracle_topk_row_nnz_*      Sec. 3.2's first step with Sec. 2.2's irregular
+ *   oracle_topk_row_nnz_*      Sec. 3.2's first step with Sec. 2's irregular
  *                              pruning: each row's count of the K weights of
  *                              largest magnitude (the row density)
  *   oracle_assign_block_sizes  Sec. 3.2 (density-adaptive rounding rule)
@@ -48,7 +48,7 @@ int oracle_set_threads(int n) {
 }
 
 /* ------------------------------------------------------------------------ */
-/* Sec. 3.2 starts from the mask of irregular pruning (Sec. 2.2: keep the K
+/* Sec. 3.2 starts from the mask of irregular pruning (Sec. 2, "Irregular Pruning": keep the K
  * weights of largest magnitude) and only counts it: row r's density is its
  * number of kept weights over cols.  Here: sort all magnitudes (widened
  * exactly to double) in decreasing order, take the K-th one as the threshold t,

@@ -1,6 +1,7 @@
 // assign.cu -- the row densities of Sec. 3.2's first step on the GPU: each
 // row's count of the K weights of largest magnitude (the mask of irregular
-// pruning, Sec. 2.2, used only to measure density).
+// pruning, Sec. 2 "Irregular Pruning and Index Decoding", used only to
+// measure density).
 //
 // The K-th largest magnitude is found by radix selection over the stored
 // magnitude bits (15 for bf16, 31 for fp32: |w| orders like its bits for every
