@@ -1,11 +1,13 @@
 // spmm.cu -- y = W_darb X on the GPU (Sec. 3.2, Fig. 6(b)): the entry the C
-// ABI calls.  Batch <= 4 runs the row-per-lane kernel (rowlane.cuh: the
-// HBM-bound regime, values and offsets stream once), wider batches the
+// ABI calls.  Batch 1 runs the one-group-per-CTA kernel (gemv.cuh) when x fits
+// in shared memory, batch <= 4 otherwise the row-per-lane kernel (rowlane.cuh:
+// the HBM-bound regime, values and offsets stream once), wider batches the
 // batch-per-lane kernel (batch.cuh, instantiated in spmm_batch.cu) or, for
 // bf16 weights from kTensorCoreMinBatch columns on, the tensor-core kernel
 // (tc.cuh, in spmm_tc.cu).  All accumulate in fp32, add partial sums in a
 // fixed order (results are deterministic) and write every output element
 // exactly once.
+#include "gemv.cuh"
 #include "rowlane.cuh"
 
 #include <mutex>
@@ -20,6 +22,9 @@ cudaError_t launch_spmm(const Format &f, const float *X, int64_t ldx, int64_t ba
         const cudaError_t e = launch_spmm_tc(f, X, ldx, batch, Y, ldy, early, stream);
         if (e != cudaErrorNotSupported) return e;
     }
+    if (batch == 1 && f.cols <= int64_t(gemv::kMaxCols))
+        return f.bf16 ? gemv::launch<true>(f, X, ldx, Y, ldy, early, stream)
+                      : gemv::launch<false>(f, X, ldx, Y, ldy, early, stream);
     if (batch <= 4) {
         const RnnArgs none{};
         return f.bf16 ? rowlane::launch_any<true, kModeY>(f, X, ldx, batch, Y, ldy, none, early, stream)
