@@ -73,26 +73,46 @@ def measured_bf16_tflops():
         return FALLBACK_BF16_TFLOPS, "fallback"
 
 
-def library_source_hash() -> str:
-    """sha1 over the library's CUDA sources: identifies the kernels a profile was taken on."""
+# The CUDA sources each profiled call's kernels are built from (the shared
+# headers included): a summary stays valid while these files are unchanged.
+_COMMON_SOURCES = ("darb_internal.h", "launch.cuh", "tma.cuh", "spmm.cu")
+_CALL_SOURCES = {
+    "encode": ("encode.cu",),
+    "b1": ("gemv.cuh", "kernels_common.cuh"),
+    "b16": ("batch.cuh", "kernels_common.cuh", "rnn_epilogue.cuh", "spmm_batch.cu"),
+    "tc": ("tc.cuh", "tcgen05.cuh", "spmm_tc.cu"),
+}
+
+
+def call_sources(call: str):
+    """The csrc files the kernels of a bench call (e.g. fc6_spmm_b256) come from."""
+    if call.endswith("_encode"):
+        kind = "encode"
+    else:
+        b = int(call.rsplit("_b", 1)[1])
+        kind = "b1" if b == 1 else ("b16" if b < 33 else "tc")
+    return tuple(sorted(_COMMON_SOURCES + _CALL_SOURCES[kind]))
+
+
+def library_source_hash(call: str) -> str:
+    """sha1 over the CUDA sources of a call's kernels: identifies the kernels a profile was taken on."""
     import hashlib
     csrc = os.path.join(ROOT, "paper_1911_08020_gb300", "csrc")
     h = hashlib.sha1()
-    for name in sorted(os.listdir(csrc)):
-        if name.endswith((".cu", ".cuh", ".h")):
-            with open(os.path.join(csrc, name), "rb") as f:
-                h.update(name.encode() + b"\0" + f.read())
+    for name in call_sources(call):
+        with open(os.path.join(csrc, name), "rb") as f:
+            h.update(name.encode() + b"\0" + f.read())
     return h.hexdigest()[:12]
 
 
 def profiled_traffic(call: str):
     """DRAM bytes per launch of `call` from the committed ncu summaries under
     profiles/ (lines 'traffic: <call> <bytes> src=<hash>'), or None when no
-    summary was taken on the current kernels."""
+    summary was taken on the current sources of the call's kernels."""
     pdir = os.path.join(ROOT, "profiles")
     if not os.path.isdir(pdir):
         return None
-    want = library_source_hash()
+    want = library_source_hash(call)
     for name in sorted(os.listdir(pdir)):
         if not name.endswith((".md", ".txt")):
             continue
