@@ -16,7 +16,8 @@
 // column).  A NaN anywhere in a block would be that block's largest magnitude,
 // so checking each block's winner finds every NaN at no extra cost.
 //
-// Scan: each thread takes one block.  Blocks are m words apart, so a straight
+// Scan: each thread takes one block (for bf16 with power-of-two m >= 8, in
+// 16-byte units of 8 elements, see the kernel).  Blocks are m words apart, so a straight
 // scan makes lanes collide on shared-memory banks whenever m is even; each lane
 // instead starts at a rotated position s(lane) = (lane * 2^a) / 32,
 // a = min(v2(m), 5), and wraps around.  Lanes that share a bank offset
@@ -164,6 +165,17 @@ encode_kernel(EncodeTarget t, const void *W, int64_t ldw, int32_t *status, int s
         const int mw = m >> 1;
         const int aw = mw > 0 ? min(__ffs(mw) - 1, 5) : 0;
         const int rotw = (lane << aw) >> 5;
+        // bf16, m a power of two >= 8 and a 16-byte aligned tile: 16-byte units of
+        // 8 elements (U = m / 8 per block).  Per unit, the largest magnitude by
+        // packed 16-bit maxima (no per-element key); per block, the unit that
+        // first reaches the block's largest magnitude (ties to the lowest unit,
+        // through the unit number in the key); then, in that unit alone, the
+        // lowest element with that magnitude.  Lanes start at rotated units
+        // (lane & 7 for U >= 8, else (lane & 7) * U / 8: a quarter-warp's 16-byte
+        // loads then meet 8 distinct bank groups) and run all U units (no divergence).
+        const int U = m >> 3;
+        const bool units = BF16 && m >= 8 && (m & (m - 1)) == 0 && (g.off0 % 16 == 0);
+        const int rotu = !units ? 0 : U >= 8 ? (lane & 7) : ((lane & 7) * U) >> 3;
         for (int base = 0; base < nb; base += kEncThreads) {
             const int jj = base + tid;
             uint32_t best_o = 0;
@@ -172,7 +184,29 @@ encode_kernel(EncodeTarget t, const void *W, int64_t ldw, int32_t *status, int s
                 int o = rot;
                 if constexpr (BF16) {
                     uint32_t best = 0;
-                    if (pairs) {
+                    if (units) {
+                        const uint4 *ublk = reinterpret_cast<const uint4 *>(blk);
+                        const uint32_t umsk = uint32_t(U) - 1u;
+                        uint32_t ukey = 0;   // (largest magnitude << 16) | (0xFFFF - unit)
+#pragma unroll 4
+                        for (int k = 0; k < U; ++k) {
+                            const uint32_t u = (uint32_t(rotu) + uint32_t(k)) & umsk;
+                            const uint4 q = ublk[u];
+                            const uint32_t m01 = __vmaxu2(q.x & 0x7FFF7FFFu, q.y & 0x7FFF7FFFu);
+                            const uint32_t m23 = __vmaxu2(q.z & 0x7FFF7FFFu, q.w & 0x7FFF7FFFu);
+                            const uint32_t mm = __vmaxu2(m01, m23);
+                            const uint32_t mx = max(mm >> 16, mm & 0xFFFFu);   // the unit's largest magnitude
+                            ukey = max(ukey, (mx << 16) | (0xFFFFu - u));
+                        }
+                        const uint32_t mag = ukey >> 16, u = 0xFFFFu - (ukey & 0xFFFFu);
+                        const uint4 q = ublk[u];
+                        const uint32_t w[4] = {q.x, q.y, q.z, q.w};
+                        uint32_t first = 8;   // lowest element of the unit with that magnitude
+#pragma unroll
+                        for (int j = 7; j >= 0; --j)
+                            if (((w[j >> 1] >> (16 * (j & 1))) & 0x7FFFu) == mag) first = uint32_t(j);
+                        best = (mag << 16) | (0xFFFFu - (8u * u + first));
+                    } else if (pairs) {
                         const uint32_t *wblk = reinterpret_cast<const uint32_t *>(blk);
                         int qw = rotw;
 #pragma unroll 2
