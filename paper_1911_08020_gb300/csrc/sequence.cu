@@ -34,6 +34,8 @@ constexpr int kSeqWarps = kThreads / 32;
 constexpr int kMaxCtas = 256;
 constexpr size_t kSmemCap = 226 * 1024;   // dynamic shared memory, below the 227 KB opt-in with room for the static part
 constexpr int kMaxTile = 32;              // batch columns per tile, at most (one per lane)
+constexpr int kClusterFourSlack = 0;      // SMs given up for clusters of four instead of pairs, at most
+                                          // (measured on the RNN workloads: four saved L2 reads but not time)
 constexpr size_t kCellOnChip = 16 * 1024; // LSTM cell state kept in shared memory up to this size
 
 struct Ranges {
@@ -51,8 +53,8 @@ struct SeqArgs {
     int ipad, hpad;
     // tensor-map staging (tma != 0): boxes of {bt columns, bxh rows} over x_t
     // (nbx of them) and {bt, bhh} over h_{t-1} (nbh), tile_bytes per tile in all;
-    // with cs = 2 the two CTAs of a cluster each load half of the boxes and
-    // multicast them to both
+    // with cs = 2 or 4 the CTAs of a cluster each load 1/cs of the boxes and
+    // multicast them to all
     int tma, cs, nbx, bxh, nbh, bhh;
     uint32_t tile_bytes;
     int64_t B;
@@ -434,7 +436,9 @@ seq_kernel(Format f, SeqArgs a, Ranges rg, SmemPlan sp, const __grid_constant__ 
                         float *dst = s_in + (int64_t(isx ? y : a.ipad + y) << lbt);
                         const CUtensorMap *m = isx ? &mx : (t == 0 ? &mh0 : &mhs);
                         const int z = isx ? t : (t == 0 ? 0 : t - 1);
-                        if (cs > 1) tensor3d_g2s_multicast(dst, m, static_cast<int>(b0), y, z, &s_full, 3);
+                        if (cs > 1)
+                            tensor3d_g2s_multicast(dst, m, static_cast<int>(b0), y, z, &s_full,
+                                                   static_cast<uint16_t>((1u << cs) - 1u));
                         else tensor3d_g2s(dst, m, static_cast<int>(b0), y, z, &s_full);
                     }
                     ok = mbar_wait(&s_full, tile & 1, false);
@@ -526,6 +530,35 @@ seq_kernel(Format f, SeqArgs a, Ranges rg, SmemPlan sp, const __grid_constant__ 
 
 namespace {
 
+// Clusters of `cs` CTAs of the sequence kernel that fit on the device at once
+// with the largest shared memory a launch may ask for (the GPCs decide how many
+// clusters of a size can be placed).
+template <bool BF16, int MODE>
+int cluster_capacity(int cs) {
+    static int cache[5] = {};
+    if (cache[cs] != 0) return cache[cs] > 0 ? cache[cs] : 0;
+    cudaFuncSetAttribute(seq::seq_kernel<BF16, MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                         static_cast<int>(seq::kSmemCap));
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeClusterDimension;
+    at[0].val.clusterDim.x = static_cast<unsigned>(cs);
+    at[0].val.clusterDim.y = 1;
+    at[0].val.clusterDim.z = 1;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(static_cast<unsigned>(cs));
+    cfg.blockDim = dim3(seq::kThreads);
+    cfg.dynamicSmemBytes = seq::kSmemCap;
+    cfg.attrs = at;
+    cfg.numAttrs = 1;
+    int n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, seq::seq_kernel<BF16, MODE>, &cfg) != cudaSuccess) {
+        cudaGetLastError();
+        n = 0;
+    }
+    cache[cs] = n > 0 ? n : -1;
+    return n > 0 ? n : 0;
+}
+
 // Contiguous unit ranges over G CTAs with about equal kept weights each.
 // Returns the largest weight count and unit count of any CTA.
 void split_units(const std::vector<int64_t> &kept, int G, seq::Ranges &rg, int64_t &kept_cap, int &units_cap) {
@@ -604,7 +637,21 @@ static cudaError_t launch_seq_t(const Format &f, const int32_t *row_m, seq::SeqA
     // tensor-map staging needs 16-byte rows of every source (B a multiple of 4)
     const bool tma_ok = ptrs && B % 4 == 0 && tensor_map_encoder() != nullptr;
     int G = std::max(1, std::min({sm_count(), H, kMaxCtas}));
-    if (tma_ok && G >= 2) G &= ~1;   // clusters of two CTAs share each staged tile
+    // clusters of cs CTAs share each staged tile (each CTA loads 1/cs of it and
+    // multicasts): four when GPCs place almost as many CTAs in clusters of four
+    // as in pairs, else two
+    int want_cs = 1;
+    if (tma_ok && G >= 2) {
+        const int g2 = std::min(G, 2 * cluster_capacity<BF16, MODE>(2)) & ~1;
+        const int g4 = std::min(G, 4 * cluster_capacity<BF16, MODE>(4)) & ~3;
+        if (g4 >= 4 && g4 + kClusterFourSlack >= g2) {
+            want_cs = 4;
+            G = g4;
+        } else if (g2 >= 2) {
+            want_cs = 2;
+            G = g2;
+        }
+    }
     Ranges rg{};
     int64_t kept_cap = 0;
     int units_cap = 0;
@@ -659,7 +706,7 @@ static cudaError_t launch_seq_t(const Format &f, const int32_t *row_m, seq::SeqA
     a.lbt = 0;
     while ((1 << a.lbt) < bt) ++a.lbt;
     a.tma = tma_ok && bt >= 4 ? 1 : 0;
-    a.cs = a.tma && G % 2 == 0 ? 2 : 1;
+    a.cs = a.tma ? want_cs : 1;
     if (a.tma) {
         a.nbx = nbx;
         a.bxh = bxh;
@@ -706,7 +753,7 @@ static cudaError_t launch_seq_t(const Format &f, const int32_t *row_m, seq::SeqA
     at[0].id = cudaLaunchAttributeCooperative;
     at[0].val.cooperative = 1;
     at[1].id = cudaLaunchAttributeClusterDimension;
-    at[1].val.clusterDim.x = 2;
+    at[1].val.clusterDim.x = static_cast<unsigned>(std::max(a.cs, 1));
     at[1].val.clusterDim.y = 1;
     at[1].val.clusterDim.z = 1;
     cudaLaunchConfig_t cfg = {};
@@ -716,16 +763,16 @@ static cudaError_t launch_seq_t(const Format &f, const int32_t *row_m, seq::SeqA
     cfg.stream = stream;
     cfg.attrs = at;
     cfg.numAttrs = 1;
-    if (a.cs == 2) {   // clusters of two, if that many pairs fit at once
+    if (a.cs > 1) {   // clusters, if that many fit at once with this launch's shared memory
         cfg.numAttrs = 2;
         cfg.attrs = at + 1;
-        int pairs = 0;
-        if (cudaOccupancyMaxActiveClusters(&pairs, seq_kernel<BF16, MODE>, &cfg) != cudaSuccess || 2 * pairs < G) {
+        int n = 0;
+        if (cudaOccupancyMaxActiveClusters(&n, seq_kernel<BF16, MODE>, &cfg) != cudaSuccess || a.cs * n < G) {
             cudaGetLastError();
             a.cs = 1;
         }
         cfg.attrs = at;
-        cfg.numAttrs = a.cs == 2 ? 2 : 1;
+        cfg.numAttrs = a.cs > 1 ? 2 : 1;
     }
     // workspace: barrier word and abort flag; the cell state when it is neither
     // on chip nor in c_last; the x parts and the product input they come from
