@@ -36,7 +36,7 @@
 namespace darb {
 namespace {
 
-constexpr int kEncThreads = 256;
+constexpr int kEncThreads = 128;   // small CTAs: more of them (and their copies) per SM; 256 was 5-17% slower
 
 // Bytes of one stage: the largest tile of the handle plus room for its
 // 16-byte-misaligned start, in 128-byte units.  Sizing the ring to the
