@@ -130,35 +130,54 @@ __device__ __forceinline__ void split2(float a, float b, uint32_t *hi, uint32_t 
     *lo = *reinterpret_cast<const uint32_t *>(&l);
 }
 
-// hi, lo: cols x batch bf16 with row pitch ldw (a multiple of 8).  Each thread
-// takes four consecutive batch columns of one row.
+// hi, lo: cols x batch bf16 with row pitch ldw (a multiple of 8).  Item i is
+// four consecutive batch columns of one row; a thread takes kSplitItems items
+// a gridDim.x * 256 apart and issues all their loads before it converts any
+// (one round trip to HBM instead of one per item).  cols * ceil(batch / 4)
+// < 2^30 (checked by the caller), so no item index overflows an int.
+constexpr int kSplitItems = 4;
 __global__ void __launch_bounds__(256)
 split_kernel(const float *X, int64_t ldx, int64_t batch, int64_t cols, uint16_t *hi, uint16_t *lo, int64_t ldw,
              int *arrive, int narrive) {
     pdl_launch_dependents();
     pdl_wait_previous();   // X may come from the previous kernel; the workspace may still be read by it
     for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < narrive; i += gridDim.x * blockDim.x) arrive[i] = 0;
-    const int64_t q4 = (batch + 3) / 4;
+    const int q4 = static_cast<int>((batch + 3) / 4), nb = static_cast<int>(batch);
+    const int items = static_cast<int>(cols) * q4;
     const bool vec = (ldx & 3) == 0 && (reinterpret_cast<uintptr_t>(X) & 15) == 0;
-    for (int64_t i = int64_t(blockIdx.x) * blockDim.x + threadIdx.x; i < cols * q4;
-         i += int64_t(gridDim.x) * blockDim.x) {
-        const int64_t k = i / q4, b = (i - k * q4) * 4;
-        const float *x = X + k * ldx + b;
-        float4 v;
-        if (vec && b + 4 <= batch) {
-            v = __ldg(reinterpret_cast<const float4 *>(x));
-        } else {
-            v.x = __ldg(x);
-            v.y = b + 1 < batch ? __ldg(x + 1) : 0.0f;
-            v.z = b + 2 < batch ? __ldg(x + 2) : 0.0f;
-            v.w = b + 3 < batch ? __ldg(x + 3) : 0.0f;
+    const int stride = gridDim.x * blockDim.x;
+    for (int i0 = blockIdx.x * blockDim.x + threadIdx.x; i0 < items; i0 += kSplitItems * stride) {
+        float4 v[kSplitItems];
+#pragma unroll
+        for (int u = 0; u < kSplitItems; ++u) {
+            const int i = i0 + u * stride;
+            v[u] = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+            if (i < items) {
+                const int k = i / q4, b = (i - k * q4) * 4;
+                const float *x = X + int64_t(k) * ldx + b;
+                if (vec && b + 4 <= nb) {
+                    v[u] = __ldg(reinterpret_cast<const float4 *>(x));
+                } else {
+                    v[u].x = __ldg(x);
+                    if (b + 1 < nb) v[u].y = __ldg(x + 1);
+                    if (b + 2 < nb) v[u].z = __ldg(x + 2);
+                    if (b + 3 < nb) v[u].w = __ldg(x + 3);
+                }
+            }
         }
-        uint2 h, l;
-        split2(v.x, v.y, &h.x, &l.x);
-        split2(v.z, v.w, &h.y, &l.y);
-        // ldw is a multiple of 8 and b of 4, so b + 4 <= ldw: 8-byte aligned, inside the row
-        *reinterpret_cast<uint2 *>(hi + k * ldw + b) = h;
-        *reinterpret_cast<uint2 *>(lo + k * ldw + b) = l;
+#pragma unroll
+        for (int u = 0; u < kSplitItems; ++u) {
+            const int i = i0 + u * stride;
+            if (i < items) {
+                const int k = i / q4, b = (i - k * q4) * 4;
+                uint2 h, l;
+                split2(v[u].x, v[u].y, &h.x, &l.x);
+                split2(v[u].z, v[u].w, &h.y, &l.y);
+                // ldw is a multiple of 8 and b of 4, so b + 4 <= ldw: 8-byte aligned, inside the row
+                *reinterpret_cast<uint2 *>(hi + int64_t(k) * ldw + b) = h;
+                *reinterpret_cast<uint2 *>(lo + int64_t(k) * ldw + b) = l;
+            }
+        }
     }
 }
 
@@ -664,7 +683,13 @@ cudaError_t launch_kw(const Format &f, const float *X, int64_t ldx, int64_t batc
         return cudaErrorNotSupported;
     }
     const int64_t items = f.cols * ((batch + 3) / 4);
-    const unsigned sgrid = static_cast<unsigned>(std::min<int64_t>((items + 255) / 256, int64_t(sm_count()) * 8));
+    if (items >= (int64_t(1) << 30)) {   // 16 GB of X and more: the CUDA-core path
+        cudaFreeAsync(ws, stream);
+        return cudaErrorNotSupported;
+    }
+    const int64_t per_cta = 256 * kSplitItems;
+    const unsigned sgrid = static_cast<unsigned>(std::max<int64_t>(1, std::min<int64_t>((items + per_cta - 1) / per_cta,
+                                                                                      int64_t(sm_count()) * 8)));
     e = launch_ex(split_kernel, dim3(sgrid), dim3(256), 0, stream, 1, true, X, ldx, batch, f.cols, hi, lo, ldw,
                   arrive, static_cast<int>(counters / 4));
     if (e == cudaSuccess && coop) {
