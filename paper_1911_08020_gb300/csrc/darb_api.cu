@@ -263,7 +263,8 @@ Format format_of(const darb_handle_s *h) {
     }
     f.ngroups = static_cast<int32_t>(h->groups.size());
     f.bf16 = h->wtype == DARB_BF16 ? 1 : 0;
-    f.m_max = h->groups.empty() ? 1 : h->groups.back().m;
+    f.m_max = h->groups.empty() ? 1 : h->groups.back().m;   // groups are sorted by block size
+    f.m_min = h->groups.empty() ? 1 : h->groups.front().m;
     f.rows = h->rows;
     f.cols = h->cols;
     return f;

@@ -59,6 +59,7 @@ struct Format {
     int32_t ngroups;
     int32_t bf16;            // value dtype: 0 fp32, 1 bf16
     int32_t m_max;           // largest block size of any row
+    int32_t m_min;           // smallest block size of any row (0: unknown)
     int64_t rows, cols;
 };
 

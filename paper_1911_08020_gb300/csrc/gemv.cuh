@@ -14,8 +14,16 @@
 // a row meet in shared memory and are added in warp order (deterministic).
 //
 // Compared with the row-per-lane kernel (rowlane.cuh) it needs no cluster,
-// no distributed shared memory and no per-round staging of the values: a
-// group costs one round trip to HBM for its data and one for x.
+// no distributed shared memory and no per-round staging of the values.
+//
+// gemv_bulk_kernel is the same product with the whole group in shared memory:
+// at the start one thread bulk-copies the group's values and offsets (one
+// contiguous run each) and, once the previous kernel is done, x; the warps
+// then read their chunks from shared memory.  Every byte of a call is in
+// flight after one issue, so a call costs one round trip to HBM (the W copies
+// even start while the previous kernel drains), where the register kernel
+// needs one per batch of chunks plus one for x.  It is used when the largest
+// group and x fit in shared memory and the arrays are 16-byte aligned.
 #pragma once
 
 #include "kernels_common.cuh"
@@ -142,9 +150,100 @@ gemv_kernel(Format f, const float *X, int64_t ldx, float *Y, int64_t ldy, int ea
     }
 }
 
+// Shared memory of gemv_bulk_kernel: [0, 128) the two mbarriers, then vcap
+// bytes for a group's values, ocap for its offsets, then x.
+template <bool BF16>
+__global__ void __launch_bounds__(kThreadsG)
+gemv_bulk_kernel(Format f, const float *X, int64_t ldx, float *Y, int64_t ldy, int early, int vcap, int ocap) {
+    constexpr int kEsz = BF16 ? 2 : 4;
+    extern __shared__ __align__(128) unsigned char sm[];
+    uint64_t *bar = reinterpret_cast<uint64_t *>(sm);   // [0]: values and offsets, [1]: x
+    unsigned char *const s_val = sm + 128;
+    uint32_t *const s_off = reinterpret_cast<uint32_t *>(s_val + vcap);
+    float *const s_x = reinterpret_cast<float *>(reinterpret_cast<unsigned char *>(s_off) + ocap);
+    __shared__ float s_part[kWarpsG][kSlots];
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int gi = blockIdx.x;
+    const Group g = f.groups[gi];
+    const int nch = (g.n + kChunk - 1) / kChunk;
+    const uint32_t vbytes = uint32_t(nch) * kSlots * kChunk * kEsz;
+    const uint32_t obytes = uint32_t(nch) * kSlots * (g.nib ? 4u : 8u);
+    const int64_t cols = f.cols;
+    // x in one copy when it is one aligned run of whole 16-byte units
+    const bool xbulk = ldx == 1 && (reinterpret_cast<uintptr_t>(X) & 15) == 0 && (cols & 3) == 0;
+    auto copy_w = [&] {
+        mbar_arrive_expect_tx(&bar[0], vbytes + obytes);
+        bulk_g2s(s_val, static_cast<const unsigned char *>(f.vals) + g.val_off * kEsz, vbytes, &bar[0]);
+        bulk_g2s(s_off, f.offs + g.off_off, obytes, &bar[0]);
+    };
+
+    pdl_launch_dependents();
+    if (tid == 0) {
+        mbar_init(&bar[0], 1);
+        mbar_init(&bar[1], 1);
+        fence_mbar_init();
+        if (early) copy_w();   // the handle's data never changes after encoding
+    }
+    pdl_wait_previous();   // x may come from the previous kernel, and Y may still be read by it
+    if (tid == 0) {
+        if (!early) copy_w();
+        if (xbulk) {
+            mbar_arrive_expect_tx(&bar[1], uint32_t(cols) * 4u);
+            bulk_g2s(s_x, X, uint32_t(cols) * 4u, &bar[1]);
+        }
+    }
+    if (!xbulk)
+        for (int64_t k = tid; k < cols; k += kThreadsG) s_x[k] = __ldg(X + k * ldx);
+    __syncthreads();   // the barriers' initialisation and the plain copy of x are seen by all threads
+    const bool ok = __syncthreads_and(mbar_wait(&bar[0], 0) && (!xbulk || mbar_wait(&bar[1], 0)));
+    float acc = 0.0f;
+    if (ok) {
+        for (int c = warp; c < nch; c += kWarpsG) {
+            const int rec = c * kSlots + lane;
+            ChunkData<BF16> d;
+            if constexpr (BF16) {
+                d.v[0] = reinterpret_cast<const uint4 *>(s_val)[rec];
+            } else {
+                d.v[0] = reinterpret_cast<const uint4 *>(s_val)[2 * rec];
+                d.v[1] = reinterpret_cast<const uint4 *>(s_val)[2 * rec + 1];
+            }
+            d.o = g.nib ? make_uint2(s_off[rec], 0u) : reinterpret_cast<const uint2 *>(s_off)[rec];
+            acc += chunk_dot<BF16>(g, c, d, s_x);
+        }
+    } else if (tid == 0) {
+        atomicOr(f.status, kStatusTimeout);
+    }
+    s_part[warp][lane] = acc;
+    __syncthreads();
+    if (ok && warp == 0 && lane < g.nrows) {
+        float sum = 0.0f;
+#pragma unroll
+        for (int w = 0; w < kWarpsG; ++w) sum += s_part[w][lane];
+        Y[int64_t(f.rowmap[gi * kSlots + lane]) * ldy] = sum;
+    }
+}
+
+constexpr size_t kBulkSmemLimit = 225 * 1024;   // dynamic: 227 KB a block, less the static partial sums
+
 template <bool BF16>
 cudaError_t launch(const Format &f, const float *X, int64_t ldx, float *Y, int64_t ldy, bool early,
                    cudaStream_t stream) {
+    // the largest group is one of the smallest block size
+    if (f.m_min > 0 && (reinterpret_cast<uintptr_t>(f.vals) & 15) == 0 &&
+        (reinterpret_cast<uintptr_t>(f.offs) & 15) == 0) {
+        const int64_t nch = ((f.cols + f.m_min - 1) / f.m_min + kChunk - 1) / kChunk;
+        const int64_t vcap = nch * kSlots * kChunk * (BF16 ? 2 : 4);
+        // any group (m >= m_min) has at most nch chunks; room for 8-byte offset
+        // records, which groups of m > 16 use
+        const int64_t ocap = nch * kSlots * 8;
+        const int64_t smem = 128 + vcap + ocap + f.cols * 4;
+        if (smem <= int64_t(kBulkSmemLimit)) {
+            static const cudaError_t attr = allow_smem(gemv_bulk_kernel<BF16>, kBulkSmemLimit);
+            if (attr != cudaSuccess) return attr;
+            return launch_ex(gemv_bulk_kernel<BF16>, dim3(static_cast<unsigned>(f.ngroups)), dim3(kThreadsG),
+                             size_t(smem), stream, 1, true, f, X, ldx, Y, ldy, early ? 1 : 0, int(vcap), int(ocap));
+        }
+    }
     const size_t smem = size_t(f.cols) * 4;
     static const cudaError_t attr = allow_smem(gemv_kernel<BF16>, kMaxCols * 4);
     if (attr != cudaSuccess) return attr;
