@@ -13,8 +13,9 @@
 //    stream-ordered workspace (the tensor cores take bf16 X only with bf16
 //    weights, and one bf16 copy would be too coarse);
 //  * tc_kernel.  Work unit: 256 rows (eight consecutive 32-row groups, any
-//    block sizes) x one batch tile of N = 32..256 columns x one cluster
-//    rank's share of the columns of W, walked in stages of 32 columns:
+//    block sizes) x one batch tile of N = 32..256 columns x one split-K
+//    rank's share of the columns of W, walked in stages of 32 columns (64
+//    for N <= 64):
 //      - a TMA warp copies the stage's rows of hi and lo for the batch tile
 //        straight into two MN-major B tiles (128-byte swizzle; rows and
 //        columns past the ends read as zeros);
@@ -28,12 +29,14 @@
 //      - an MMA warp issues, per stage and 128-row half, A*B_hi + A*B_lo for
 //        two K=16 steps into that half's TMEM accumulator (128 lanes x N fp32
 //        columns) and releases the stage with tcgen05.commit.
-//    At the end the ranks of a cluster add their partial accumulators: every
+//    At the end the ranks of a tile add their partial accumulators: every
 //    rank writes its partial tile to workspace (L2-resident, coalesced),
-//    the cluster meets at one barrier, and each rank adds the partials of
-//    its slice of the rows in rank order (deterministic) and writes them to
-//    Y.  (Pushing the rows through distributed shared memory instead moved
-//    only ~10 bytes/clock per SM.)
+//    the ranks meet -- on the tile's arrival counter (bounded wait) when they
+//    are CTAs of one cooperative launch, at a cluster barrier when they are
+//    a cluster -- and each rank adds the partials of its slice of the rows
+//    in rank order (deterministic) and writes them to Y.  (Pushing the rows
+//    through distributed shared memory instead moved only ~10 bytes/clock
+//    per SM.)
 // Per stage the shared memory moves the MMA operands (96 KB at N = 256), the
 // copied B tiles and the A rows; with the split done beforehand that stays
 // near what the tensor cores need for the stage's multiplies.
