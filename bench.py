@@ -141,14 +141,88 @@ def call_name(kind, mi, b):
 
 
 # ----------------------------------------------------------------------------- clocks
+def pci_bus_id(torch, device: int):
+    """domain:bus:device.0 of a CUDA device (hex), or None where torch does not report it."""
+    p = torch.cuda.get_device_properties(device)
+    try:
+        return f"{p.pci_domain_id:x}:{p.pci_bus_id:x}:{p.pci_device_id:x}.0"
+    except AttributeError:
+        return None
+
+
+class NvmlPoller:
+    """SM clock and clock-event reasons read through NVML (the driver's
+    libnvidia-ml, read-only queries) every ~0.5 ms from a thread while the
+    timed region runs: a region of a few milliseconds is far shorter than
+    nvidia-smi's sampling period.  Inert where NVML is missing."""
+    CLOCK_SM = 1
+    # clock-event reason bits of NVML's public header
+    REASONS = {0x4: "sw_power_cap", 0x8: "hw_slowdown", 0x20: "sw_thermal_slowdown", 0x40: "hw_thermal_slowdown"}
+
+    def __init__(self, index: int, pci: str | None = None):
+        import ctypes
+        self.c = ctypes
+        self.samples = []
+        self.lib = self.dev = None
+        self.max_mhz = None
+        self.stop = threading.Event()
+        try:
+            lib = ctypes.CDLL("libnvidia-ml.so.1")
+            if lib.nvmlInit_v2() != 0:
+                return
+            dev = ctypes.c_void_p()
+            # the GPU CUDA runs on, by PCI address (CUDA and NVML may number devices differently)
+            found = pci is not None and lib.nvmlDeviceGetHandleByPciBusId_v2(pci.encode(), ctypes.byref(dev)) == 0
+            if not found and lib.nvmlDeviceGetHandleByIndex_v2(ctypes.c_uint(index), ctypes.byref(dev)) != 0:
+                lib.nvmlShutdown()
+                return
+            mx = ctypes.c_uint()
+            if lib.nvmlDeviceGetMaxClockInfo(dev, ctypes.c_int(self.CLOCK_SM), ctypes.byref(mx)) == 0:
+                self.max_mhz = float(mx.value)
+            self.reasons_fn = getattr(lib, "nvmlDeviceGetCurrentClocksEventReasons", None) or \
+                getattr(lib, "nvmlDeviceGetCurrentClocksThrottleReasons", None)
+            self.lib, self.dev = lib, dev
+        except (OSError, AttributeError):
+            self.lib = None
+
+    def _poll(self):
+        c = self.c
+        clk, rs = c.c_uint(), c.c_ulonglong()
+        while not self.stop.is_set():
+            if self.lib.nvmlDeviceGetClockInfo(self.dev, c.c_int(self.CLOCK_SM), c.byref(clk)) == 0:
+                mask = rs.value if (self.reasons_fn is not None and self.reasons_fn(self.dev, c.byref(rs)) == 0) else 0
+                self.samples.append((float(clk.value), int(mask)))
+            time.sleep(0.0005)
+
+    def __enter__(self):
+        if self.lib is not None:
+            self.thread = threading.Thread(target=self._poll, daemon=True)
+            self.thread.start()
+        return self
+
+    def __exit__(self, *exc):
+        if self.lib is not None:
+            self.stop.set()
+            self.thread.join(timeout=5)
+            self.lib.nvmlShutdown()
+
+    def summary(self):
+        if not self.samples:
+            return None
+        reasons = sorted({name for _, m in self.samples for bit, name in self.REASONS.items() if m & bit})
+        return {"sm_mhz": statistics.median(v for v, _ in self.samples), "sm_max_mhz": self.max_mhz,
+                "reasons": reasons, "samples": len(self.samples), "source": "nvml, during the timed region"}
+
+
 class ClockSampler:
-    """nvidia-smi samples of SM clock and throttle reasons while the timed region runs."""
+    """nvidia-smi samples of SM clock and throttle reasons around the timed region
+    (used when NVML cannot be read; a short region may see none of its own)."""
     FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
               "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
               "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
 
-    def __init__(self, index: int):
-        self.index = index
+    def __init__(self, index):
+        self.index = index   # an nvidia-smi -i argument: index or PCI bus id
         self.proc = None
         self.lines = []
 
@@ -195,7 +269,7 @@ class ClockSampler:
         if not sm:
             return None
         return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
-                "samples": len(sm)}
+                "samples": len(sm), "source": "nvidia-smi, around the timed region"}
 
 
 # ----------------------------------------------------------------------------- distributed
@@ -393,12 +467,14 @@ def run_gpu(args, world, rank, local):
     end = torch.cuda.Event(enable_timing=True)
     barrier(world)
     torch.cuda.synchronize()
-    with ClockSampler(local) as clk:
-        start.record(stream)
-        for s in range(args.steps):
-            step_graphs[s % NSETS].replay()
-        end.record(stream)
-        torch.cuda.synchronize()
+    pci = pci_bus_id(torch, local)
+    with ClockSampler(pci or local) as clk:
+        with NvmlPoller(local, pci) as nv:
+            start.record(stream)
+            for s in range(args.steps):
+                step_graphs[s % NSETS].replay()
+            end.record(stream)
+            torch.cuda.synchronize()
     barrier(world)
     elapsed_ms = start.elapsed_time(end)
     wl.check_encode()
@@ -421,7 +497,7 @@ def run_gpu(args, world, rank, local):
         per_call[i] = a.elapsed_time(b) / (reps * NSETS)
     wl.check_encode()
     peak, peak_kind = measured_peaks()
-    clocks = clk.summary()
+    clocks = nv.summary() or clk.summary()
     sm_mhz = (clocks or {}).get("sm_mhz") or 2070.0
     nsm = torch.cuda.get_device_properties(torch.cuda.current_device()).multi_processor_count
     # on-chip gather bound: every (kept weight, batch column) product reads its
