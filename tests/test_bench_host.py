@@ -99,3 +99,23 @@ def test_traffic_lines_parse(name):
             # a line taken on the current sources is the one the bench reports
             if parts[3] == f"src={bench.library_source_hash(call)}":
                 assert bench.profiled_traffic(call) == int(parts[2])
+
+
+def test_nvml_reason_bits_name_the_rejecting_reasons():
+    p = bench.NvmlPoller.__new__(bench.NvmlPoller)   # no NVML needed: summarise given samples
+    p.max_mhz = 2070.0
+    p.samples = [(2070.0, 0x0), (2055.0, 0x4), (1900.0, 0x8 | 0x40), (2070.0, 0x1)]
+    s = p.summary()
+    assert s["reasons"] == ["hw_slowdown", "hw_thermal_slowdown", "sw_power_cap"]
+    assert s["sm_mhz"] == pytest.approx(2062.5) and s["sm_max_mhz"] == 2070.0 and s["samples"] == 4
+    p.samples = []
+    assert p.summary() is None
+
+
+def test_nvidia_smi_lines_parse():
+    c = bench.ClockSampler(0)
+    c.lines = ["2070, 2070, 900.5, 0x0000000000000000, Not Active, Not Active, Not Active, Not Active",
+               "1980, 2070, 1390.0, 0x0000000000000004, Not Active, Not Active, Not Active, Active",
+               "garbage"]
+    s = c.summary()
+    assert s["reasons"] == ["sw_power_cap"] and s["samples"] == 2 and s["sm_mhz"] == pytest.approx(2025.0)
