@@ -150,9 +150,16 @@ DARB_API darb_status_t darb_sync_status(darb_handle_t h, cudaStream_t stream);
  *   X  device fp32, cols x batch, ldx >= batch, 4-byte aligned.
  *   Y  device fp32, rows x batch, ldy >= batch; overwritten.  Must not
  *      overlap X.
- * Accumulates in fp32.  Asynchronous on `stream`; allocates nothing; the
- * handle is only read, so calls on several streams may share it.
- * Errors: DARB_ERR_INVALID_ARG (null, batch <= 0, ld < batch); DARB_ERR_CUDA.
+ * Accumulates in fp32.  Asynchronous on `stream`; the handle is only read, so
+ * calls on several streams may share it.  For bf16 weights from 33 batch
+ * columns on it runs the tensor-core kernels (darb_spmm_ex, DARB_PATH_AUTO),
+ * which take their workspace from the device's stream-ordered memory pool on
+ * `stream` for the duration of the call; otherwise it allocates nothing.  A
+ * bounded device wait that gave up is reported by darb_sync_status.
+ * Errors: DARB_ERR_INVALID_ARG (null, batch <= 0, ld < batch, X or Y not
+ * 4-byte aligned, Y overlapping X); DARB_ERR_UNSUPPORTED (batch above 2^19);
+ * DARB_ERR_OOM (the pool could not supply the tensor-core workspace);
+ * DARB_ERR_CUDA.
  */
 DARB_API darb_status_t darb_spmm(darb_handle_t h, const float *X, int64_t ldx, int64_t batch, float *Y,
                         int64_t ldy, cudaStream_t stream);
