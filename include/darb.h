@@ -24,14 +24,15 @@
  *    and any scratch it allocates, and releases both in darb_destroy.
  *  - Work is enqueued on the caller's stream.  Only darb_encode, darb_import,
  *    darb_export, darb_sync_status, darb_rnn_reserve and darb_destroy
- *    synchronise; the product, step and sequence calls are asynchronous and
- *    allocate nothing beyond the RNN step scratch and the pool scratch noted
- *    below.
- *  - Scratch that a call takes from the device's stream-ordered memory pool
- *    (the tensor-core product, the sequence calls) is returned to the pool on
- *    the same stream.  The first such call on a device raises the release
- *    threshold of the device's current pool to 1 GiB if it is lower, so that
- *    freed scratch stays mapped across synchronisations.
+ *    synchronise; the product, step and sequence calls are asynchronous.
+ *    darb_spmm allocates nothing; the step calls use scratch owned by the
+ *    handle (darb_rnn_reserve sizes it up front).
+ *  - Only two opt-in calls take scratch from the device's stream-ordered
+ *    memory pool: darb_spmm_ex with DARB_PATH_TENSOR_CORES and the sequence
+ *    calls.  They return it to the pool on the same stream.  The first such
+ *    call on a device raises the release threshold of the device's current
+ *    pool to 1 GiB if it is lower, so that freed scratch stays mapped across
+ *    synchronisations; darb_spmm never touches the pool.
  *  - There is no CPU fallback: without a usable CUDA device the GPU calls
  *    return DARB_ERR_CUDA.
  */
@@ -60,7 +61,7 @@ typedef enum {
     DARB_ERR_NONFINITE = 2,     /* a NaN weight was found while encoding                 */
     DARB_ERR_OOM = 3,           /* a device or host allocation failed                    */
     DARB_ERR_CUDA = 4,          /* a CUDA runtime call or kernel launch failed           */
-    DARB_ERR_TIMEOUT = 5,       /* a bounded device-side wait gave up (reserved)         */
+    DARB_ERR_TIMEOUT = 5,       /* a bounded device-side wait gave up (darb_sync_status)  */
     DARB_ERR_UNSUPPORTED = 6    /* arguments valid but not supported by these kernels    */
 } darb_status_t;
 
@@ -139,7 +140,8 @@ DARB_API darb_status_t darb_reencode(darb_handle_t h, const void *W, int64_t ldw
 
 /* Synchronise `stream` and report what the handle's kernels recorded on the
  * device since the last call, then clear it: DARB_ERR_TIMEOUT if a bounded
- * wait for a bulk copy gave up (results of that call are not valid), else
+ * device wait (for a bulk copy, or at a sequence call's grid barrier) gave up
+ * -- results of that call are not valid, the device stays usable -- else
  * DARB_ERR_NONFINITE if a (re)encode met a NaN, else DARB_OK.                */
 DARB_API darb_status_t darb_sync_status(darb_handle_t h, cudaStream_t stream);
 
@@ -150,15 +152,14 @@ DARB_API darb_status_t darb_sync_status(darb_handle_t h, cudaStream_t stream);
  *   X  device fp32, cols x batch, ldx >= batch, 4-byte aligned.
  *   Y  device fp32, rows x batch, ldy >= batch; overwritten.  Must not
  *      overlap X.
- * Accumulates in fp32.  Asynchronous on `stream`; the handle is only read, so
- * calls on several streams may share it.  For bf16 weights from 33 batch
- * columns on it runs the tensor-core kernels (darb_spmm_ex, DARB_PATH_AUTO),
- * which take their workspace from the device's stream-ordered memory pool on
- * `stream` for the duration of the call; otherwise it allocates nothing.  A
- * bounded device wait that gave up is reported by darb_sync_status.
+ * Every kept weight is multiplied only by the activation its block selects
+ * (a NaN or infinity in an activation row that no kept weight selects does
+ * not reach Y), in fp32, on the CUDA cores, for every dtype and batch.
+ * Asynchronous on `stream`; allocates nothing; the handle is only read, so
+ * calls on several streams may share it.  A bounded device wait that gave up
+ * is reported by darb_sync_status.
  * Errors: DARB_ERR_INVALID_ARG (null, batch <= 0, ld < batch, X or Y not
  * 4-byte aligned, Y overlapping X); DARB_ERR_UNSUPPORTED (batch above 2^19);
- * DARB_ERR_OOM (the pool could not supply the tensor-core workspace);
  * DARB_ERR_CUDA.
  */
 DARB_API darb_status_t darb_spmm(darb_handle_t h, const float *X, int64_t ldx, int64_t batch, float *Y,
@@ -167,15 +168,15 @@ DARB_API darb_status_t darb_spmm(darb_handle_t h, const float *X, int64_t ldx, i
 /* Which kernels compute a product (the paper has no counterpart: these are two
  * ways of evaluating the same sum on the GPU).                               */
 typedef enum {
-    DARB_PATH_AUTO = 0,          /* what darb_spmm does                              */
+    DARB_PATH_AUTO = 0,          /* what darb_spmm does: the CUDA-core gather        */
     DARB_PATH_CUDA_CORES = 1,    /* gather-multiply-add on the CUDA cores (any weights) */
     DARB_PATH_TENSOR_CORES = 2   /* densified tiles on the tensor cores (bf16 weights) */
 } darb_path_t;
 
 /*
- * darb_spmm with the kernel family chosen by the caller.  DARB_PATH_AUTO uses
- * the tensor cores for bf16 weights from 33 batch columns on, else the CUDA
- * cores.  The tensor-core path multiplies every activation
+ * darb_spmm with the kernel family chosen by the caller.  DARB_PATH_AUTO and
+ * DARB_PATH_CUDA_CORES are darb_spmm.  DARB_PATH_TENSOR_CORES is an opt-in
+ * alternative that is not the paper's per-block selection: it multiplies every activation
  * of a stage by the densified tile, zeros included, with X split into two
  * bf16 parts (x = hi + lo): |Y - exact| <= 2^-16 * sum |val * x| plus fp32
  * rounding, a NaN or infinity in X may make rows NaN that do not select it,
@@ -190,9 +191,9 @@ typedef enum {
 DARB_API darb_status_t darb_spmm_ex(darb_handle_t h, const float *X, int64_t ldx, int64_t batch, float *Y,
                                     int64_t ldy, darb_path_t path, cudaStream_t stream);
 
-/* The kernel family darb_spmm takes for this handle and batch (*path), and
- * how many kernels it launches per call (*kernels: 1 on the CUDA cores, 2 on
- * the tensor cores, the split of X and the product).  Host only.
+/* The kernel family darb_spmm takes for this handle and batch (*path: always
+ * DARB_PATH_CUDA_CORES), and how many kernels it launches per call (*kernels:
+ * 1).  Host only.
  * Errors: DARB_ERR_INVALID_ARG (unknown handle, batch <= 0, null outputs). */
 DARB_API darb_status_t darb_spmm_path(darb_handle_t h, int64_t batch, darb_path_t *path, int32_t *kernels);
 
@@ -254,13 +255,16 @@ DARB_API darb_status_t darb_gru_step(darb_handle_t h, int64_t I, int64_t H, int6
  * has 64 to 2^19 columns (T * B) and the workspace below stays under 1 GiB,
  * the x parts of all T steps are computed first as one product
  * W [x_0 .. x_{T-1}; 0] of T * B columns (darb_spmm's kernels and numerics,
- * the tensor cores for bf16 weights); the recurrence then stages and
+ * the CUDA-core gather); the recurrence then stages and
  * multiplies only h_{t-1}.
  * Resources: one cooperative launch of one CTA per SM (at most H CTAs); a
  * stream-ordered workspace of 256 bytes, plus H x B floats when c_last is
  * NULL and the cell state does not fit on chip, plus (I + H + 4H) x T*B
  * floats when the x parts are precomputed.  A barrier wait longer than 1 s
  * ends the launch and is reported by darb_sync_status as DARB_ERR_TIMEOUT.
+ * For testing that path, the environment variable DARB_TEST_BARRIER_TIMEOUT=1
+ * (read at every launch) shortens the limit to 1 ms and makes CTA 0 withhold
+ * its first arrival, so the launch times out on purpose.
  * Errors: DARB_ERR_INVALID_ARG (shape mismatch, null, overlap, T < 0);
  * DARB_ERR_UNSUPPORTED when a CTA's share of the decoded matrix plus one
  * column tile of [x_t; h_{t-1}] does not fit in shared memory, or cols > 65535;

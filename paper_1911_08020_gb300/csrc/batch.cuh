@@ -288,9 +288,11 @@ batch_kernel(Format f, const int2 *__restrict__ sets, const float *__restrict__ 
     };
 
     bool ok = true;
+    int issued = 0;   // rounds whose copies were started (producer warp), for the drain below
     if (warp == kConsumers) {
         // ---------------- producer warp
         const int pre = min(rounds, kStages);
+        if (early) issued = pre;
         if (early && lane == 0)
             for (int r = 0; r < pre; ++r) issue(r, r, true, false);
         pdl_wait_previous();
@@ -305,6 +307,7 @@ batch_kernel(Format f, const int2 *__restrict__ sets, const float *__restrict__ 
             }
             if (!use_tma) load_x_plain(r, st);
             if (lane == 0) issue(r, st, !(early && r < kStages), true);
+            issued = max(issued, r + 1);
         }
         if (!ok && lane == 0) atomicOr(f.status, kStatusTimeout);
     } else {
@@ -364,6 +367,15 @@ batch_kernel(Format f, const int2 *__restrict__ sets, const float *__restrict__ 
             if (lane == 0) mbar_arrive(&empty[st]);
         }
         if (!ok && lane == 0) atomicOr(f.status, kStatusTimeout);
+    }
+    if (!__syncthreads_and(ok) && warp == kConsumers && lane == 0) {
+        // a wait gave up: copies may still be landing in the stages.  Give the
+        // last round issued into each stage a second bounded wait before the
+        // stages are reused below (the sums of this call are not valid).
+        for (int st = 0; st < kStages; ++st) {
+            const int last = issued - 1 - ((issued - 1 - st) % kStages + kStages) % kStages;
+            if (last >= 0 && last < issued) mbar_wait(&full[st], (last / kStages) & 1);
+        }
     }
     __syncthreads();   // every round consumed: the stages are free for the partial sums
     // partial sums of every row slot of the set, slot-major: part[s][part][0..kBt)
@@ -487,16 +499,15 @@ inline void grid_shape_rnn(const Format &f, int64_t tiles, int *level, unsigned 
 // CTAs of one batch_kernel instantiation resident per SM (shared memory is the limit).
 template <bool BF16, int LPR, int CPL, int MODE>
 inline int resident_per_sm() {
-    static const int n = [] {
+    const auto fn = batch_kernel<BF16, LPR, CPL, MODE>;
+    return static_cast<int>(per_device(reinterpret_cast<const void *>(fn), 0, [fn] {
         int v = 0;
-        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&v, batch_kernel<BF16, LPR, CPL, MODE>, kThreads,
-                                                          smem_bytes<BF16>()) != cudaSuccess) {
+        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&v, fn, kThreads, smem_bytes<BF16>()) != cudaSuccess) {
             cudaGetLastError();
             v = 0;
         }
-        return v > 0 ? v : 1;
-    }();
-    return n;
+        return static_cast<long long>(v > 0 ? v : 1);
+    }));
 }
 
 template <bool BF16, int LPR, int CPL, int MODE>
@@ -504,7 +515,7 @@ cudaError_t launch(const Format &f, const float *X, int64_t ldx, int64_t batch, 
                    const RnnArgs &ra, bool early, cudaStream_t stream) {
     constexpr int kBt = LPR * CPL;
     constexpr size_t smem = smem_bytes<BF16>();
-    static const cudaError_t attr = allow_smem(batch_kernel<BF16, LPR, CPL, MODE>, smem);
+    const cudaError_t attr = allow_smem(batch_kernel<BF16, LPR, CPL, MODE>, smem);
     if (attr != cudaSuccess) return attr;
     CUtensorMap xmap, hmap;
     std::memset(&xmap, 0, sizeof xmap);

@@ -568,9 +568,9 @@ darb_status_t darb_assign_from_weights(const void *W, darb_dtype_t wtype, int64_
 
 darb_status_t darb_spmm_path(darb_handle_t h, int64_t batch, darb_path_t *path, int32_t *kernels) {
     if (!live(h) || batch <= 0 || path == nullptr || kernels == nullptr) return DARB_ERR_INVALID_ARG;
-    const bool tensor = h->wtype == DARB_BF16 && batch >= darb::kTensorCoreMinBatch && batch <= kMaxBatch;
-    *path = tensor ? DARB_PATH_TENSOR_CORES : DARB_PATH_CUDA_CORES;
-    *kernels = tensor ? 2 : 1;
+    // darb_spmm always takes the CUDA-core gather: one kernel per call
+    *path = DARB_PATH_CUDA_CORES;
+    *kernels = 1;
     return DARB_OK;
 }
 

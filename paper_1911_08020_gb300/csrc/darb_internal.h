@@ -106,16 +106,11 @@ cudaError_t launch_spmm_batch(const Format &f, const float *X, int64_t ldx, int6
 cudaError_t launch_spmm_tc(const Format &f, const float *X, int64_t ldx, int64_t batch, float *Y,
                            int64_t ldy, bool early, cudaStream_t stream);
 
-// Smallest batch that the automatic choice sends to the tensor cores.  On
-// the FC6/FC7 shapes the CUDA cores win up to 32 columns (one 32-column
-// tile) and the tensor cores from 48 on; 33..47 cost the CUDA-core kernel a
-// second tile and the tensor-core kernel nothing more than 48.
-constexpr int64_t kTensorCoreMinBatch = 33;
-
 // `early`: the handle's data is known to be complete, so a kernel may start
 // reading it before the previous kernel on the stream has finished (PDL).
-// `path`: a darb_path_t.  cudaErrorNotSupported if DARB_PATH_TENSOR_CORES
-// was asked for a call the tensor-core kernel cannot take.
+// `path`: a darb_path_t; DARB_PATH_AUTO and DARB_PATH_CUDA_CORES both take the
+// CUDA-core gather.  cudaErrorNotSupported if DARB_PATH_TENSOR_CORES was asked
+// for a call the tensor-core kernel cannot take.
 cudaError_t launch_spmm(const Format &f, const float *X, int64_t ldx, int64_t batch, float *Y,
                         int64_t ldy, bool early, int path, cudaStream_t stream);
 

@@ -288,7 +288,7 @@ inline size_t encode_smem_max() {
 template <bool BF16>
 cudaError_t launch_encode_t(const EncodeTarget &t, const void *W, int64_t ldw, int32_t *status,
                             cudaStream_t stream) {
-    static const cudaError_t a = allow_smem(encode_kernel<BF16>, encode_smem_max<BF16>());
+    const cudaError_t a = allow_smem(encode_kernel<BF16>, encode_smem_max<BF16>());
     if (a != cudaSuccess) return a;
     const int sbytes = stage_bytes(t);
     const size_t smem = encode_smem<BF16>(sbytes);

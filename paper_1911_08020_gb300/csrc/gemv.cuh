@@ -211,7 +211,11 @@ gemv_bulk_kernel(Format f, const float *X, int64_t ldx, float *Y, int64_t ldy, i
             acc += chunk_dot<BF16>(g, c, d, s_x);
         }
     } else if (tid == 0) {
+        // a copy did not land in time: record it, and give the copies still in
+        // flight a second bounded wait before the CTA (and its shared memory) ends
         atomicOr(f.status, kStatusTimeout);
+        mbar_wait(&bar[0], 0);
+        if (xbulk) mbar_wait(&bar[1], 0);
     }
     s_part[warp][lane] = acc;
     __syncthreads();
@@ -238,14 +242,14 @@ cudaError_t launch(const Format &f, const float *X, int64_t ldx, float *Y, int64
         const int64_t ocap = nch * kSlots * 8;
         const int64_t smem = 128 + vcap + ocap + f.cols * 4;
         if (smem <= int64_t(kBulkSmemLimit)) {
-            static const cudaError_t attr = allow_smem(gemv_bulk_kernel<BF16>, kBulkSmemLimit);
+            const cudaError_t attr = allow_smem(gemv_bulk_kernel<BF16>, kBulkSmemLimit);
             if (attr != cudaSuccess) return attr;
             return launch_ex(gemv_bulk_kernel<BF16>, dim3(static_cast<unsigned>(f.ngroups)), dim3(kThreadsG),
                              size_t(smem), stream, 1, true, f, X, ldx, Y, ldy, early ? 1 : 0, int(vcap), int(ocap));
         }
     }
     const size_t smem = size_t(f.cols) * 4;
-    static const cudaError_t attr = allow_smem(gemv_kernel<BF16>, kMaxCols * 4);
+    const cudaError_t attr = allow_smem(gemv_kernel<BF16>, kMaxCols * 4);
     if (attr != cudaSuccess) return attr;
     return launch_ex(gemv_kernel<BF16>, dim3(static_cast<unsigned>(f.ngroups)), dim3(kThreadsG), smem, stream, 1, true,
                      f, X, ldx, Y, ldy, early ? 1 : 0);

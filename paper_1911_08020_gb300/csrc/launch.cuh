@@ -7,9 +7,52 @@
 #include <cudaTypedefs.h>
 #include <cuda_runtime.h>
 
+#include <map>
+#include <mutex>
+#include <tuple>
 #include <utility>
 
 namespace darb {
+
+// The calling thread's current device (0 if it cannot be read).
+inline int current_device() {
+    int d = 0;
+    if (cudaGetDevice(&d) != cudaSuccess) {
+        cudaGetLastError();
+        d = 0;
+    }
+    return d;
+}
+
+namespace detail {
+inline std::mutex &cache_mutex() {
+    static std::mutex mu;
+    return mu;
+}
+// (key, sub-key, device) -> value
+inline std::map<std::tuple<const void *, long long, int>, long long> &cache_map() {
+    static std::map<std::tuple<const void *, long long, int>, long long> m;
+    return m;
+}
+}  // namespace detail
+
+// A figure computed once per (key, sub-key, device) and kept for the process:
+// kernel attributes and occupancy belong to a device, so a process that
+// drives several devices computes them on each.  `compute` runs outside the
+// lock (it may call the runtime); two threads may both compute a missing entry.
+template <class F>
+long long per_device(const void *key, long long sub, F compute) {
+    const auto k = std::make_tuple(key, sub, current_device());
+    {
+        std::lock_guard<std::mutex> lk(detail::cache_mutex());
+        const auto it = detail::cache_map().find(k);
+        if (it != detail::cache_map().end()) return it->second;
+    }
+    const long long v = compute();
+    std::lock_guard<std::mutex> lk(detail::cache_mutex());
+    detail::cache_map()[k] = v;
+    return v;
+}
 
 template <typename... KArgs, typename... Args>
 cudaError_t launch_ex(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
@@ -38,12 +81,24 @@ cudaError_t launch_ex(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t sm
     return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
 }
 
-// Raise a kernel's dynamic shared memory limit once (per process).
+// Raise a kernel's dynamic shared memory limit to at least `bytes` on the
+// current device (once per kernel, device and larger size).
 template <typename... KArgs>
 cudaError_t allow_smem(void (*kernel)(KArgs...), size_t bytes) {
     if (bytes <= 48 * 1024) return cudaSuccess;
-    return cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                static_cast<int>(bytes));
+    const void *fn = reinterpret_cast<const void *>(kernel);
+    const auto k = std::make_tuple(fn, -1ll, current_device());
+    std::lock_guard<std::mutex> lk(detail::cache_mutex());
+    auto &m = detail::cache_map();
+    const auto it = m.find(k);
+    if (it != m.end() && it->second >= static_cast<long long>(bytes)) return cudaSuccess;
+    const cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(bytes));
+    if (e != cudaSuccess) {
+        cudaGetLastError();
+        return e;
+    }
+    m[k] = static_cast<long long>(bytes);
+    return cudaSuccess;
 }
 
 // cuTensorMapEncodeTiled from the driver (through the runtime, so that the

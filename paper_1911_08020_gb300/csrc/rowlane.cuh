@@ -262,7 +262,7 @@ template <bool BF16, int BT, int MODE>
 cudaError_t launch(const Format &f, const float *X, int64_t ldx, int64_t batch, float *Y, int64_t ldy,
                    const RnnArgs &ra, bool early, cudaStream_t stream) {
     constexpr size_t smem = smem_bytes<BF16, BT, MODE>();
-    static const cudaError_t attr = allow_smem(rowlane_kernel<BF16, BT, MODE>, smem);
+    const cudaError_t attr = allow_smem(rowlane_kernel<BF16, BT, MODE>, smem);
     if (attr != cudaSuccess) return attr;
     const unsigned ksc = cluster_size(f);
     const dim3 grid(static_cast<unsigned>(f.ngroups) * ksc);

@@ -17,13 +17,15 @@
 // barrier (arrival counter in global memory, spun on with a 1 s limit; on
 // expiry the kernel records a timeout, raises an abort flag that ends every
 // other CTA's wait, and returns).  The launch is cooperative, so all CTAs are
-// resident and the barrier cannot starve.
+// resident and the barrier cannot starve.  No CTA touches another CTA's shared
+// memory, and no CTA leaves while a copy it issued may still be landing.
 #include "darb_internal.h"
 #include "launch.cuh"
 #include "rnn_epilogue.cuh"
 #include "tma.cuh"
 
 #include <algorithm>
+#include <cstdlib>
 #include <vector>
 
 namespace darb {
@@ -34,8 +36,6 @@ constexpr int kSeqWarps = kThreads / 32;
 constexpr int kMaxCtas = 256;
 constexpr size_t kSmemCap = 226 * 1024;   // dynamic shared memory, below the 227 KB opt-in with room for the static part
 constexpr int kMaxTile = 32;              // batch columns per tile, at most (one per lane)
-constexpr int kClusterFourSlack = 0;      // SMs given up for clusters of four instead of pairs, at most
-                                          // (measured on the RNN workloads: four saved L2 reads but not time)
 constexpr size_t kCellOnChip = 16 * 1024; // LSTM cell state kept in shared memory up to this size
 
 struct Ranges {
@@ -52,10 +52,8 @@ struct SeqArgs {
     // h_{t-1} from row ipad, a zero row at ipad + hpad
     int ipad, hpad;
     // tensor-map staging (tma != 0): boxes of {bt columns, bxh rows} over x_t
-    // (nbx of them) and {bt, bhh} over h_{t-1} (nbh), tile_bytes per tile in all;
-    // with cs = 2 or 4 the CTAs of a cluster each load 1/cs of the boxes and
-    // multicast them to all
-    int tma, cs, nbx, bxh, nbh, bhh;
+    // (nbx of them) and {bt, bhh} over h_{t-1} (nbh), tile_bytes per tile in all
+    int tma, nbx, bxh, nbh, bhh;
     uint32_t tile_bytes;
     int64_t B;
     const float *gx;        // x parts of the gate sums of every step, rows x ldgx (row r, step t, column b
@@ -74,6 +72,8 @@ struct SeqArgs {
     unsigned *bar;          // arrival counter, zero at launch
     int *abort_flag;        // zero at launch
     int32_t *status;
+    unsigned long long barrier_ns;   // time limit of a grid-barrier wait (kWaitLimitNs unless a test shortens it)
+    int skip_cta;           // test hook: this CTA does not arrive at the first barrier (-1: none)
 };
 
 // Byte offsets of the regions of a CTA's dynamic shared memory.
@@ -128,7 +128,7 @@ __device__ __forceinline__ bool grid_barrier(const SeqArgs &a, unsigned target, 
     __syncthreads();
     if (threadIdx.x == 0) {
         __threadfence();   // the CTA's h_t stores are visible before its arrival counts
-        atomicAdd(a.bar, 1u);
+        if (!(int(blockIdx.x) == a.skip_cta && target == gridDim.x)) atomicAdd(a.bar, 1u);
         int ok = 1;
         const unsigned long long t0 = global_timer_ns();
         for (unsigned spin = 0;; ++spin) {
@@ -140,7 +140,7 @@ __device__ __forceinline__ bool grid_barrier(const SeqArgs &a, unsigned target, 
                     ok = 0;
                     break;
                 }
-                if (global_timer_ns() - t0 > kWaitLimitNs) {
+                if (global_timer_ns() - t0 > a.barrier_ns) {
                     ok = 0;
                     atomicExch(a.abort_flag, 1);
                     atomicOr(a.status, kStatusTimeout);
@@ -296,7 +296,7 @@ seq_kernel(Format f, SeqArgs a, Ranges rg, SmemPlan sp, const __grid_constant__ 
     using PT = typename P::T;
     extern __shared__ __align__(16) unsigned char sm[];
     __shared__ int s_ok, s_nitems, s_staged, s_next;
-    __shared__ __align__(8) uint64_t s_full, s_empty;   // tile landed; every CTA of the cluster done with it
+    __shared__ __align__(8) uint64_t s_full;   // the staged tile has landed
     PT *s_w = reinterpret_cast<PT *>(sm + sp.w_off);
     int *s_rowptr = reinterpret_cast<int *>(sm + sp.rowptr_off);
     int *s_mid = reinterpret_cast<int *>(sm + sp.mid_off);          // GRU: first kept weight of a row on h
@@ -321,10 +321,6 @@ seq_kernel(Format f, SeqArgs a, Ranges rg, SmemPlan sp, const __grid_constant__ 
     // GRU without precomputed x parts keeps the x and h sums of each item apart
     const bool split = kGru && !pre;
     const int kin = a.ipad + a.hpad;
-    // the cluster this CTA actually runs in: multicast and remote arrivals only
-    // when the launch really formed clusters of a.cs CTAs
-    const int cs = a.cs > 1 && cluster_nctarank() == uint32_t(a.cs) ? a.cs : 1;
-    const uint32_t rank = cs > 1 ? cluster_ctarank() : 0;
     auto grow = [&](int lr) { return (lr / nu) * H + u0 + lr % nu; };
 
     // ---- prologue: row sizes, biases, cell state, the zero row of the staged input
@@ -348,10 +344,8 @@ seq_kernel(Format f, SeqArgs a, Ranges rg, SmemPlan sp, const __grid_constant__ 
     for (int j = tid; j < bt; j += kThreads) s_in[(kin << lbt) + j] = 0.0f;
     if (tid == 0) {
         mbar_init(&s_full, 1);
-        mbar_init(&s_empty, cs);
         fence_mbar_init();
     }
-    if (cs > 1) cluster_sync_all();   // the partner's barriers exist before anything targets them
     __syncthreads();
     // row pointers and work items: every row cut into pieces of at most a.piece weights
     if (tid == 0) {
@@ -413,7 +407,7 @@ seq_kernel(Format f, SeqArgs a, Ranges rg, SmemPlan sp, const __grid_constant__ 
     __syncthreads();
 
     // ---- the steps
-    int tile = 0;   // tiles staged so far: the parity of both barriers
+    int tile = 0;   // tiles staged so far: the parity of s_full
     float *c_run = kGru ? nullptr : (a.c_on_chip ? s_c : a.c_state + int64_t(u0) * B);
     for (int t = 0; t < a.T; ++t) {
         const float *xt = a.x + int64_t(t) * I * B;
@@ -425,27 +419,26 @@ seq_kernel(Format f, SeqArgs a, Ranges rg, SmemPlan sp, const __grid_constant__ 
             const int nb = static_cast<int>(B - b0 < bt ? B - b0 : bt);
             // stage [x_t; h_{t-1}] (or h_{t-1}) for columns [b0, b0 + nb), zeros past the batch
             if (a.tma && tid == 0) {
-                // every CTA of the cluster is done with the previous tile
-                bool ok = tile == 0 || mbar_wait_cluster(&s_empty, (tile - 1) & 1);
-                if (ok) {
-                    fence_proxy_async_global();   // h_{t-1} was published by generic stores
-                    mbar_arrive_expect_tx(&s_full, a.tile_bytes);
-                    for (int bx = static_cast<int>(rank); bx < a.nbx + a.nbh; bx += cs) {
-                        const bool isx = bx < a.nbx;
-                        const int y = isx ? bx * a.bxh : (bx - a.nbx) * a.bhh;
-                        float *dst = s_in + (int64_t(isx ? y : a.ipad + y) << lbt);
-                        const CUtensorMap *m = isx ? &mx : (t == 0 ? &mh0 : &mhs);
-                        const int z = isx ? t : (t == 0 ? 0 : t - 1);
-                        if (cs > 1)
-                            tensor3d_g2s_multicast(dst, m, static_cast<int>(b0), y, z, &s_full,
-                                                   static_cast<uint16_t>((1u << cs) - 1u));
-                        else tensor3d_g2s(dst, m, static_cast<int>(b0), y, z, &s_full);
-                    }
-                    ok = mbar_wait(&s_full, tile & 1, false);
+                // every thread of this CTA is done with the previous tile (the
+                // barrier that ended it); order those reads before the copies
+                fence_proxy_async_smem();
+                fence_proxy_async_global();   // h_{t-1} was published by generic stores
+                mbar_arrive_expect_tx(&s_full, a.tile_bytes);
+                for (int bx = 0; bx < a.nbx + a.nbh; ++bx) {
+                    const bool isx = bx < a.nbx;
+                    const int y = isx ? bx * a.bxh : (bx - a.nbx) * a.bhh;
+                    float *dst = s_in + (int64_t(isx ? y : a.ipad + y) << lbt);
+                    const CUtensorMap *m = isx ? &mx : (t == 0 ? &mh0 : &mhs);
+                    const int z = isx ? t : (t == 0 ? 0 : t - 1);
+                    tensor3d_g2s(dst, m, static_cast<int>(b0), y, z, &s_full);
                 }
+                bool ok = mbar_wait(&s_full, tile & 1, false);
                 if (!ok) {
                     atomicOr(a.status, kStatusTimeout);
                     atomicExch(a.abort_flag, 1);
+                    // the copies may still land: give them a second bounded wait
+                    // before this CTA leaves
+                    mbar_wait(&s_full, tile & 1, false);
                 }
                 s_staged = ok;
             }
@@ -512,15 +505,10 @@ seq_kernel(Format f, SeqArgs a, Ranges rg, SmemPlan sp, const __grid_constant__ 
                 }
             }
             __syncthreads();
-            if (a.tma && tid == 0)   // this CTA is done with the tile: tell every CTA of the cluster
-                for (int r = 0; r < cs; ++r) mbar_arrive_cluster(&s_empty, static_cast<uint32_t>(r));
             ++tile;
         }
         if (t + 1 < a.T && !grid_barrier(a, unsigned(t + 1) * gridDim.x, &s_ok)) return;
     }
-    // the partner's last arrival on this CTA's barrier has landed before it leaves
-    if (a.tma && cs > 1 && tid == 0 && !mbar_wait_cluster(&s_empty, (tile - 1) & 1))
-        atomicOr(a.status, kStatusTimeout);
     if constexpr (!kGru)
         if (a.c_on_chip && a.c_last)
             for (int i = tid; i < nu * B; i += kThreads) a.c_last[int64_t(u0) * B + i] = s_c[i];
@@ -530,33 +518,19 @@ seq_kernel(Format f, SeqArgs a, Ranges rg, SmemPlan sp, const __grid_constant__ 
 
 namespace {
 
-// Clusters of `cs` CTAs of the sequence kernel that fit on the device at once
-// with the largest shared memory a launch may ask for (the GPCs decide how many
-// clusters of a size can be placed).
-template <bool BF16, int MODE>
-int cluster_capacity(int cs) {
-    static int cache[5] = {};
-    if (cache[cs] != 0) return cache[cs] > 0 ? cache[cs] : 0;
-    cudaFuncSetAttribute(seq::seq_kernel<BF16, MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                         static_cast<int>(seq::kSmemCap));
-    cudaLaunchAttribute at[1];
-    at[0].id = cudaLaunchAttributeClusterDimension;
-    at[0].val.clusterDim.x = static_cast<unsigned>(cs);
-    at[0].val.clusterDim.y = 1;
-    at[0].val.clusterDim.z = 1;
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(static_cast<unsigned>(cs));
-    cfg.blockDim = dim3(seq::kThreads);
-    cfg.dynamicSmemBytes = seq::kSmemCap;
-    cfg.attrs = at;
-    cfg.numAttrs = 1;
-    int n = 0;
-    if (cudaOccupancyMaxActiveClusters(&n, seq::seq_kernel<BF16, MODE>, &cfg) != cudaSuccess) {
-        cudaGetLastError();
-        n = 0;
+// Test hook for the failure path of the grid barrier.  With the environment
+// variable DARB_TEST_BARRIER_TIMEOUT=1 a launch's barrier waits give up after
+// 1 ms and CTA 0 withholds its arrival at the first barrier: every CTA's wait
+// runs out, the launch records DARB_ERR_TIMEOUT (read by darb_sync_status),
+// raises the abort flag and ends.  Only the barrier is affected -- no copy is
+// in flight while a CTA waits there -- and the results of that call are not
+// valid.  Read on every launch so that a test can set and clear it.
+void sequence_test_hook(unsigned long long *barrier_ns, int *skip_cta) {
+    const char *v = std::getenv("DARB_TEST_BARRIER_TIMEOUT");
+    if (v != nullptr && v[0] == '1' && v[1] == '\0') {
+        *barrier_ns = 1000000ull;
+        *skip_cta = 0;
     }
-    cache[cs] = n > 0 ? n : -1;
-    return n > 0 ? n : 0;
 }
 
 // Contiguous unit ranges over G CTAs with about equal kept weights each.
@@ -636,22 +610,7 @@ static cudaError_t launch_seq_t(const Format &f, const int32_t *row_m, seq::SeqA
     const bool ptrs = (xrows == 0 || aligned(a.x)) && aligned(a.h0) && aligned(a.h_seq);
     // tensor-map staging needs 16-byte rows of every source (B a multiple of 4)
     const bool tma_ok = ptrs && B % 4 == 0 && tensor_map_encoder() != nullptr;
-    int G = std::max(1, std::min({sm_count(), H, kMaxCtas}));
-    // clusters of cs CTAs share each staged tile (each CTA loads 1/cs of it and
-    // multicasts): four when GPCs place almost as many CTAs in clusters of four
-    // as in pairs, else two
-    int want_cs = 1;
-    if (tma_ok && G >= 2) {
-        const int g2 = std::min(G, 2 * cluster_capacity<BF16, MODE>(2)) & ~1;
-        const int g4 = std::min(G, 4 * cluster_capacity<BF16, MODE>(4)) & ~3;
-        if (g4 >= 4 && g4 + kClusterFourSlack >= g2) {
-            want_cs = 4;
-            G = g4;
-        } else if (g2 >= 2) {
-            want_cs = 2;
-            G = g2;
-        }
-    }
+    const int G = std::max(1, std::min({sm_count(), H, kMaxCtas}));
     Ranges rg{};
     int64_t kept_cap = 0;
     int units_cap = 0;
@@ -706,7 +665,6 @@ static cudaError_t launch_seq_t(const Format &f, const int32_t *row_m, seq::SeqA
     a.lbt = 0;
     while ((1 << a.lbt) < bt) ++a.lbt;
     a.tma = tma_ok && bt >= 4 ? 1 : 0;
-    a.cs = a.tma ? want_cs : 1;
     if (a.tma) {
         a.nbx = nbx;
         a.bxh = bxh;
@@ -722,9 +680,7 @@ static cudaError_t launch_seq_t(const Format &f, const int32_t *row_m, seq::SeqA
     a.stage_mode = kStageScalar;
     if (ptrs && B % 4 == 0 && bt % 4 == 0) a.stage_mode = kStageQuadCols;
     else if (ptrs && B == 1 && xrows % 4 == 0 && H % 4 == 0) a.stage_mode = kStageQuadRows;
-    static const cudaError_t attr = cudaFuncSetAttribute(seq_kernel<BF16, MODE>,
-                                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                         static_cast<int>(kSmemCap));
+    const cudaError_t attr = allow_smem(seq_kernel<BF16, MODE>, kSmemCap);
     if (attr != cudaSuccess) return attr;
     // tensor maps of the staged sources: 3-D (batch, rows, step) so that a box
     // running past the last row of a step reads zeros, never the next step
@@ -744,18 +700,13 @@ static cudaError_t launch_seq_t(const Format &f, const int32_t *row_m, seq::SeqA
         if (ok && nbx) ok = make(&mx, a.x, I, T, bxh);
         if (!ok) {   // plain loads instead (the plan above has room for either)
             a.tma = 0;
-            a.cs = 1;
             a.ipad = xrows;
             a.hpad = H;
         }
     }
-    cudaLaunchAttribute at[2];
+    cudaLaunchAttribute at[1];
     at[0].id = cudaLaunchAttributeCooperative;
     at[0].val.cooperative = 1;
-    at[1].id = cudaLaunchAttributeClusterDimension;
-    at[1].val.clusterDim.x = static_cast<unsigned>(std::max(a.cs, 1));
-    at[1].val.clusterDim.y = 1;
-    at[1].val.clusterDim.z = 1;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(static_cast<unsigned>(G));
     cfg.blockDim = dim3(kThreads);
@@ -763,17 +714,11 @@ static cudaError_t launch_seq_t(const Format &f, const int32_t *row_m, seq::SeqA
     cfg.stream = stream;
     cfg.attrs = at;
     cfg.numAttrs = 1;
-    if (a.cs > 1) {   // clusters, if that many fit at once with this launch's shared memory
-        cfg.numAttrs = 2;
-        cfg.attrs = at + 1;
-        int n = 0;
-        if (cudaOccupancyMaxActiveClusters(&n, seq_kernel<BF16, MODE>, &cfg) != cudaSuccess || a.cs * n < G) {
-            cudaGetLastError();
-            a.cs = 1;
-        }
-        cfg.attrs = at;
-        cfg.numAttrs = a.cs > 1 ? 2 : 1;
-    }
+    // every wait is bounded by kWaitLimitNs; a test may shorten the barrier's
+    // limit and hold back one CTA's first arrival (sequence_test_hook)
+    a.barrier_ns = kWaitLimitNs;
+    a.skip_cta = -1;
+    sequence_test_hook(&a.barrier_ns, &a.skip_cta);
     // workspace: barrier word and abort flag; the cell state when it is neither
     // on chip nor in c_last; the x parts and the product input they come from
     const size_t cbytes = kGru || c_on_chip || c_last ? 0 : up(size_t(H) * size_t(B) * 4);

@@ -2,12 +2,14 @@
 // ABI calls.  Batch 1 runs the one-group-per-CTA kernel (gemv.cuh) when x fits
 // in shared memory, batch <= 4 otherwise the row-per-lane kernel (rowlane.cuh:
 // the HBM-bound regime, values and offsets stream once), wider batches the
-// batch-per-lane kernel (batch.cuh, instantiated in spmm_batch.cu) or, for
-// bf16 weights from kTensorCoreMinBatch columns on, the tensor-core kernel
-// (tc.cuh, in spmm_tc.cu).  All accumulate in fp32, add partial sums in a
-// fixed order (results are deterministic) and write every output element
-// exactly once.
+// batch-per-lane kernel (batch.cuh, instantiated in spmm_batch.cu).  All of
+// them evaluate exactly the per-block selection and sum of Fig. 6(b) on the
+// CUDA cores and allocate nothing.  The tensor-core kernel (tc.cuh, in
+// spmm_tc.cu) runs only when the caller asks for it by name.  All accumulate
+// in fp32, add partial sums in a fixed order (results are deterministic) and
+// write every output element exactly once.
 #include "gemv.cuh"
+#include "launch.cuh"
 #include "rowlane.cuh"
 
 #include <mutex>
@@ -18,10 +20,6 @@ namespace darb {
 cudaError_t launch_spmm(const Format &f, const float *X, int64_t ldx, int64_t batch, float *Y,
                         int64_t ldy, bool early, int path, cudaStream_t stream) {
     if (path == DARB_PATH_TENSOR_CORES) return launch_spmm_tc(f, X, ldx, batch, Y, ldy, early, stream);
-    if (path == DARB_PATH_AUTO && f.bf16 && batch >= kTensorCoreMinBatch) {
-        const cudaError_t e = launch_spmm_tc(f, X, ldx, batch, Y, ldy, early, stream);
-        if (e != cudaErrorNotSupported) return e;
-    }
     if (batch == 1 && f.cols <= int64_t(gemv::kMaxCols))
         return f.bf16 ? gemv::launch<true>(f, X, ldx, Y, ldy, early, stream)
                       : gemv::launch<false>(f, X, ldx, Y, ldy, early, stream);
@@ -57,16 +55,15 @@ cudaError_t stream_alloc(void **p, size_t bytes, cudaStream_t stream) {
 }
 
 int sm_count() {
-    static int n = [] {
-        int dev = 0, v = 0;
-        if (cudaGetDevice(&dev) != cudaSuccess ||
-            cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) {
+    static const char key = 0;
+    return static_cast<int>(per_device(&key, 0, [] {
+        int v = 0;
+        if (cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, current_device()) != cudaSuccess || v <= 0) {
             cudaGetLastError();
-            return 148;
+            return 148ll;
         }
-        return v;
-    }();
-    return n;
+        return static_cast<long long>(v);
+    }));
 }
 
 }  // namespace darb

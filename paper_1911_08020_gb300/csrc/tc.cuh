@@ -585,9 +585,8 @@ inline int tile_width(int64_t batch) {
 // Clusters of `ksplit` CTAs of this kernel that can be resident at once (-1 if unknown).
 template <int KW>
 inline int active_clusters(int ksplit, const Plan &p) {
-    static int cache[4][9] = {};
-    const int wi = p.N == 32 ? 0 : p.N == 64 ? 1 : p.N == 128 ? 2 : 3;
-    if (cache[wi][ksplit] != 0) return cache[wi][ksplit];
+    const void *key = reinterpret_cast<const void *>(tc_kernel<KW>);
+    return static_cast<int>(per_device(key, 16ll * p.N + ksplit, [&]() -> long long {
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(ksplit * 64, 1);
     cfg.blockDim = dim3(kThreads);
@@ -604,25 +603,23 @@ inline int active_clusters(int ksplit, const Plan &p) {
         cudaGetLastError();
         n = 0;
     }
-    if (n <= 0) n = -1;
-    cache[wi][ksplit] = n;
-    return n;
+    return n > 0 ? n : -1;
+    }));
 }
 
 // CTAs of this kernel that fit on the device at once (for a cooperative launch).
 template <int KW>
 inline int64_t coop_capacity(const Plan &p) {
-    static int cache[4] = {};
-    const int wi = p.N == 32 ? 0 : p.N == 64 ? 1 : p.N == 128 ? 2 : 3;
-    if (cache[wi] == 0) {
+    const void *key = reinterpret_cast<const void *>(tc_kernel<KW>);
+    const long long n = per_device(key, -1000ll - p.N, [&]() -> long long {
         int per_sm = 0;
         if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, tc_kernel<KW>, kThreads, p.smem) != cudaSuccess) {
             cudaGetLastError();
             per_sm = 0;
         }
-        cache[wi] = per_sm > 0 ? per_sm * sm_count() : -1;
-    }
-    return cache[wi] > 0 ? cache[wi] : 0;
+        return per_sm > 0 ? static_cast<long long>(per_sm) * sm_count() : -1;
+    });
+    return n > 0 ? n : 0;
 }
 
 // Cluster split: fewest waves per unit of work, i.e. the smallest
@@ -648,7 +645,7 @@ inline int pick_split(int64_t units, int KS, const Plan &p) {
 template <int KW>
 cudaError_t launch_kw(const Format &f, const float *X, int64_t ldx, int64_t batch, float *Y, int64_t ldy, bool early,
                       const Plan &p, cudaStream_t stream) {
-    static const cudaError_t a = [] {
+    const cudaError_t a = [] {
         size_t most = 0;
         for (int w = 32; w <= 256; w *= 2)
             if (stage_width(w) == KW) most = plan_for(w).smem > most ? plan_for(w).smem : most;

@@ -108,67 +108,11 @@ __device__ __forceinline__ void tensor3d_g2s(void *dst, const void *tmap, int x,
         ::"r"(smem_addr(dst)), "l"(tmap), "r"(x), "r"(y), "r"(z), "r"(smem_addr(bar)) : "memory");
 }
 
-// The same copy delivered to every CTA of the cluster in `mask`, at the same
-// shared-memory offsets of dst and bar in each: one read of L2, several SMs fed.
-__device__ __forceinline__ void tensor3d_g2s_multicast(void *dst, const void *tmap, int x, int y, int z,
-                                                       uint64_t *bar, uint16_t mask) {
-    asm volatile(
-        "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.multicast::cluster"
-        " [%0], [%1, {%2, %3, %4}], [%5], %6;"
-        ::"r"(smem_addr(dst)), "l"(tmap), "r"(x), "r"(y), "r"(z), "r"(smem_addr(bar)), "h"(mask) : "memory");
-}
-
 // Order this thread's earlier generic-proxy view of global memory (e.g. data
 // other CTAs published through a release/acquire handshake) before its later
 // async-proxy (TMA) reads.
 __device__ __forceinline__ void fence_proxy_async_global() {
     asm volatile("fence.proxy.async.global;" ::: "memory");
-}
-
-__device__ __forceinline__ uint32_t cluster_ctarank() {
-    uint32_t r;
-    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
-    return r;
-}
-
-__device__ __forceinline__ uint32_t cluster_nctarank() {
-    uint32_t n;
-    asm volatile("mov.u32 %0, %%cluster_nctarank;" : "=r"(n));
-    return n;
-}
-
-// Every thread of every CTA of the cluster (release / acquire at cluster scope).
-__device__ __forceinline__ void cluster_sync_all() {
-    asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
-}
-
-// Arrive on the mbarrier at the same offset as `bar` in CTA `rank` of this
-// cluster (this CTA included).  Release at CTA scope only: it tells the other
-// CTA that this one has finished reading its own shared memory, and must not
-// wait for this CTA's global stores to drain.
-__device__ __forceinline__ void mbar_arrive_cluster(uint64_t *bar, uint32_t rank) {
-    uint32_t remote;
-    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(smem_addr(bar)), "r"(rank));
-    asm volatile("mbarrier.arrive.shared::cluster.b64 _, [%0];" ::"r"(remote) : "memory");
-}
-
-// mbar_wait with acquire at cluster scope: for phases completed by arrivals
-// of other CTAs of the cluster.
-__device__ __forceinline__ bool mbar_wait_cluster(uint64_t *bar, uint32_t parity) {
-    const uint32_t a = smem_addr(bar);
-    unsigned long long t0 = 0;
-    while (true) {
-        uint32_t done;
-        asm volatile(
-            "{\n .reg .pred p;\n"
-            " mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2, %3;\n"
-            " selp.u32 %0, 1, 0, p;\n}\n"
-            : "=r"(done) : "r"(a), "r"(parity), "r"(10000u) : "memory");
-        if (done) return true;
-        const unsigned long long now = global_timer_ns();
-        if (t0 == 0) t0 = now;
-        else if (now - t0 > kWaitLimitNs) return false;
-    }
 }
 
 // Programmatic dependent launch: let the next kernel on the stream start its

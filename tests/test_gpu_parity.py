@@ -214,6 +214,40 @@ def test_spmm_unselected_infinities_do_not_leak():
         darb.darb_destroy(h)
 
 
+@pytest.mark.parametrize("B", [64, 256])
+def test_spmm_fc6_bf16_unselected_nonfinite_stay_out(B):
+    """FC6 (4096 x 9216 bf16) through darb_spmm at the bench's wide batches:
+    +Inf and NaN in activation rows that no kept weight selects must not reach
+    Y (Fig. 6(b): each block contributes only the activation it selects), and
+    every output matches the oracle element by element.  Every 7th column of
+    W is zeroed so that BMWM never keeps a weight there (a block's maximum
+    magnitude is never 0 for these Gaussian weights)."""
+    wl = synth.WORKLOADS["fc6_fc7"]
+    _, stored, m = synth.matrix(wl, 0)
+    stored = stored.copy()
+    stored[:, 3::7] = 0
+    h, ref = encode_both(stored, m, wl.dtype)
+    try:
+        cols = wl.shapes[0][1]
+        used = np.zeros(cols, bool)
+        nb = ref.blk_ptr[1:] - ref.blk_ptr[:-1]
+        rows_of_block = np.repeat(np.arange(len(m)), nb)
+        j = np.arange(ref.blk_ptr[-1]) - ref.blk_ptr[rows_of_block]
+        used[j * m[rows_of_block] + ref.off] = True
+        assert (~used).sum() >= cols // 7, "the case needs unselected activation rows"
+        X = synth.activations(cols, B, seed=wl.seed + 70 + B)
+        unused = np.flatnonzero(~used)
+        X[unused[0::2], :] = np.inf
+        X[unused[1::2], :] = np.nan
+        assert darb.darb_spmm_path(h, B) == (darb.PATH_CUDA_CORES, 1)
+        Y = darb.darb_spmm(h, t(X)).cpu().numpy()
+        Yr, A = oracle.darb_spmm(ref, X, with_absdot=True)
+        assert np.isfinite(Yr).all() and np.isfinite(Y).all()
+        assert_product_close(Y, Yr, A, TOL[wl.dtype])
+    finally:
+        darb.darb_destroy(h)
+
+
 @pytest.mark.parametrize("name", list(synth.WORKLOADS))
 def test_spmm_workloads_full_size(name):
     wl = synth.WORKLOADS[name]

@@ -263,3 +263,40 @@ def test_sequence_empty_and_argument_checks():
             darb.darb_gru_sequence(h, 3, I, H, B, xs, z, None, None, hs)               # 4H rows is not a GRU
     finally:
         darb.darb_destroy(h)
+
+
+@pytest.mark.parametrize("cell,I,H,B", [("lstm", 20, 200, 8), ("lstm", 7, 33, 3), ("gru", 64, 300, 12)])
+def test_barrier_timeout_is_reported_and_the_device_stays_usable(cell, I, H, B, monkeypatch):
+    """The failure path of the sequence kernels' grid barrier, made on purpose
+    from the host: DARB_TEST_BARRIER_TIMEOUT=1 shortens the barrier's limit to
+    1 ms and holds back one CTA's first arrival, so every other CTA's wait runs
+    out (no copy is in flight at a barrier, and no wait is unbounded).  The
+    call must end, darb_sync_status must report DARB_ERR_TIMEOUT, and the next
+    call, without the hook, must be correct."""
+    g = np.random.default_rng(45)
+    gates = 4 if cell == "lstm" else 3
+    T = 4
+    stored, m = _gate_matrix(g, gates, I, H, "f32", (2, 4, 8))
+    h, ref = encode_both(stored, m, "f32")
+    try:
+        xs = synth.activations(T * I, B, seed=5).reshape(T, I, B)
+        h0 = synth.state(H, B, seed=6)
+        c0 = synth.state(H, B, seed=7)
+        hs = torch.empty((T, H, B), device=dev())
+        monkeypatch.setenv("DARB_TEST_BARRIER_TIMEOUT", "1")
+        if cell == "lstm":
+            darb.darb_lstm_sequence(h, T, I, H, B, t(xs), t(h0), t(c0), None, hs)
+        else:
+            darb.darb_gru_sequence(h, T, I, H, B, t(xs), t(h0), None, None, hs)
+        with pytest.raises(darb.DarbError) as e:
+            darb.darb_sync_status(h)
+        assert e.value.status == darb.ERR_TIMEOUT
+        monkeypatch.delenv("DARB_TEST_BARRIER_TIMEOUT")
+        darb.darb_sync_status(h)   # the status was cleared by the read
+        if cell == "lstm":
+            _check_lstm_sequence(h, ref, T, I, H, B, xs, h0, c0, None, TOL["f32"])
+        else:
+            _check_gru_sequence(h, ref, T, I, H, B, xs, h0, None, None, TOL["f32"])
+        darb.darb_sync_status(h)
+    finally:
+        darb.darb_destroy(h)

@@ -133,7 +133,7 @@ def test_tensor_path_strides_and_untouched_columns():
         darb.darb_destroy(h)
 
 
-def test_path_query_matches_the_automatic_choice():
+def test_path_query_reports_the_gather_for_every_batch():
     g = np.random.default_rng(8)
     w = (0.1 * g.standard_normal((64, 256))).astype(np.float32)
     m = np.full(64, 16, np.int32)
@@ -141,8 +141,9 @@ def test_path_query_matches_the_automatic_choice():
     h16, _ = encode_both(synth.f32_to_bf16_bits(w), m, "bf16")
     try:
         assert darb.darb_spmm_path(h32, 512) == (darb.PATH_CUDA_CORES, 1)
-        assert darb.darb_spmm_path(h16, 32) == (darb.PATH_CUDA_CORES, 1)
-        assert darb.darb_spmm_path(h16, 33) == (darb.PATH_TENSOR_CORES, 2)
+        # darb_spmm never picks the tensor cores on its own: they are opt-in
+        for B in (1, 32, 33, 64, 256, 4096):
+            assert darb.darb_spmm_path(h16, B) == (darb.PATH_CUDA_CORES, 1)
         with pytest.raises(darb.DarbError):
             darb.darb_spmm_path(h16, 0)
     finally:
