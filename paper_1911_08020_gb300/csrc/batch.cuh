@@ -1,9 +1,11 @@
 // batch.cuh -- the batch-per-lane product kernel (batch > 4), as a template
 // over its output: plain Y, or the gate sums of a fused LSTM / GRU step.
 //
-// Work unit: a row set (up to 8 consecutive 32-row groups of one block-size
-// bin, so up to 256 rows), one cluster rank's share of the blocks, and one
-// batch tile of LPR*CPL columns.  The rank's blocks are walked in rounds
+// Work unit (a WorkItem of the handle's tables): a row set (up to 8
+// consecutive 32-row groups of one block-size bin, so up to 256 rows), the
+// share of its blocks one cluster rank multiplies -- sets of small block size
+// have more blocks per row and are split over more ranks, so every CTA gets
+// about the same work -- and one batch tile of LPR*CPL columns.  The rank's blocks are walked in rounds
 // through a two-stage ring in shared memory.  A producer warp starts, per
 // round, the bulk (TMA) copies of the round's kept values and packed offsets
 // (one contiguous run per group) and the 2-D tensor-map copies of the
@@ -14,9 +16,11 @@
 // share a row and each lane owns CPL columns, interleaved so that a
 // quarter-warp reads 128 contiguous bytes of an activation row: the gathers
 // are free of bank conflicts and each kept value is reused across the tile's
-// columns from registers.  Accumulators live in registers across rounds; at
-// the end the ranks add their partial sums through distributed shared memory
-// in a fixed order (deterministic), each rank finishing a slice of the rows.
+// columns from registers.  A thread works on the same chunk of all its rows at
+// once, so the gathers of different rows overlap.  Accumulators live in
+// registers across rounds; at the end the ranks of a set add their partial
+// sums through distributed shared memory in a fixed order (deterministic),
+// each rank finishing a slice of the set's rows.
 //
 // Why row sets: an activation row staged in shared memory is selected by about
 // rows/m of the set's rows, so staging traffic per FMA is 4*m/rows bytes;
@@ -151,9 +155,66 @@ __device__ __forceinline__ void chunk(const unsigned char *s_vals, const uint32_
     }
 }
 
+// One chunk (8 blocks) of NP row slots of this thread at once (no GRU split):
+// rec[p] is the staged record of row slot p.  Blocks outer, rows inner, so the
+// activation loads of the NP rows of one block are in flight together and
+// every accumulator gets one FMA per block.
+template <bool BF16, bool NIB, bool WHOLE, bool STACKED, int NP, int KQ, int LPR>
+__device__ __forceinline__ void chunk_rows(const unsigned char *s_vals, const uint32_t *s_offs, const int *rec,
+                                           const float4 *sx4, int qd, const Round &g, int jc, int m, int row_f4,
+                                           int e_lo, int e_hi, float4 (*acc)[KQ]) {
+    constexpr int kW = BF16 ? 4 : 8;
+    uint32_t vw[NP][kW];
+    uint2 ow[NP];
+#pragma unroll
+    for (int p = 0; p < NP; ++p) {
+        const uint4 *pv = reinterpret_cast<const uint4 *>(s_vals + size_t(rec[p]) * (BF16 ? 16 : 32));
+        const uint4 w0 = pv[0];
+        vw[p][0] = w0.x; vw[p][1] = w0.y; vw[p][2] = w0.z; vw[p][3] = w0.w;
+        if constexpr (!BF16) {
+            const uint4 w1 = pv[1];
+            vw[p][4] = w1.x; vw[p][5] = w1.y; vw[p][6] = w1.z; vw[p][7] = w1.w;
+        }
+        if constexpr (NIB) ow[p] = make_uint2(s_offs[rec[p]], 0u);
+        else ow[p] = reinterpret_cast<const uint2 *>(s_offs)[rec[p]];
+    }
+    const int mstride = m * row_f4;
+    const float4 *xb = sx4 + (jc * m - g.kx0) * row_f4 + qd;
+#pragma unroll
+    for (int e = 0; e < kChunk; ++e) {
+        if (WHOLE || (e >= e_lo && e < e_hi)) {
+#pragma unroll
+            for (int p = 0; p < NP; ++p) {
+                int off;
+                if constexpr (NIB) off = int((ow[p].x >> (4 * e)) & 15u);
+                else off = int(((e < 4 ? ow[p].x : ow[p].y) >> (8 * (e & 3))) & 255u);
+                float v;
+                if constexpr (BF16) v = __uint_as_float((e & 1) ? (vw[p][e >> 1] & 0xFFFF0000u) : (vw[p][e >> 1] << 16));
+                else v = __uint_as_float(vw[p][e]);
+                const float4 *xr;
+                if constexpr (STACKED) {
+                    const int kg = (jc + e) * m + off;
+                    const int tr = kg < g.kxa ? kg - g.kx0 : g.hbase + kg - g.kxb;
+                    xr = sx4 + tr * row_f4 + qd;
+                } else {
+                    xr = xb + e * mstride + off * row_f4;
+                }
+#pragma unroll
+                for (int u = 0; u < KQ; ++u) {
+                    const float4 xv = xr[u * LPR];
+                    acc[p][u].x = fmaf(v, xv.x, acc[p][u].x);
+                    acc[p][u].y = fmaf(v, xv.y, acc[p][u].y);
+                    acc[p][u].z = fmaf(v, xv.z, acc[p][u].z);
+                    acc[p][u].w = fmaf(v, xv.w, acc[p][u].w);
+                }
+            }
+        }
+    }
+}
+
 template <bool BF16, int LPR, int CPL, int MODE>
-__global__ void __launch_bounds__(kThreads)
-batch_kernel(Format f, const int2 *__restrict__ sets, const float *__restrict__ X, int64_t ldx, int64_t batch,
+__global__ void __launch_bounds__(kThreads, 2)
+batch_kernel(Format f, const WorkItem *__restrict__ items, const float *__restrict__ X, int64_t ldx, int64_t batch,
        float *__restrict__ Y, int64_t ldy, const __grid_constant__ CUtensorMap xmap,
        const __grid_constant__ CUtensorMap hmap, RnnArgs ra, int use_tma, int early) {
     constexpr bool kStacked = MODE != kModeY;
@@ -165,6 +226,9 @@ batch_kernel(Format f, const int2 *__restrict__ sets, const float *__restrict__ 
     constexpr int kRptMax = max_set_groups<LPR, CPL>() * kSlots / (kConsumers * kRpw);
     constexpr int kBoxRows = box_rows<LPR, CPL>();
     constexpr int kEsz = BF16 ? 2 : 4;
+    // rows a thread multiplies together in the inner loop
+    constexpr int kNpg = (BF16 || kQ == 1) ? (kRptMax < 4 ? kRptMax : 4) : (kRptMax < 2 ? kRptMax : 2);
+    static_assert(kRptMax % kNpg == 0, "row passes come in whole sub-groups");
     extern __shared__ __align__(128) unsigned char sm[];
     // layout: full[kStages] empty[kStages] | X stages | values stages | offsets stages
     uint64_t *full = reinterpret_cast<uint64_t *>(sm);
@@ -177,21 +241,19 @@ batch_kernel(Format f, const int2 *__restrict__ sets, const float *__restrict__ 
     cg::cluster_group cluster = cg::this_cluster();
     const int ksc = static_cast<int>(cluster.num_blocks());
     const int q = static_cast<int>(cluster.block_rank());
-    const int2 set = sets[blockIdx.x / ksc];
-    const int ng = set.y;
-    const Group g0 = f.groups[set.x];
+    const WorkItem item = items[blockIdx.x];
+    const int ng = item.ng;   // 0: an idle rank, it only joins the cluster barriers
+    const int gfirst = item.g0;
+    const Group g0 = f.groups[gfirst];
     const int m = g0.m, n = g0.n, rw = g0.nib ? 1 : 2;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int64_t b0 = int64_t(blockIdx.y) * kBt;
     const int split = kStacked ? ra.I : int(f.cols);   // first activation row of the h part
-    const int nch = (n + kChunk - 1) / kChunk;
-    const int cpc = (nch + ksc - 1) / ksc;
-    const int c0 = min(nch, q * cpc), c1 = min(nch, c0 + cpc);
-    const int J0 = c0 * kChunk, J1 = min(n, c1 * kChunk);
+    const int J0 = item.c0 * kChunk, J1 = min(n, item.c1 * kChunk);
     // blocks per round: bounded by the activation tile and by the staged records
     const int rows_cap = kXcapB / kBt - (kStacked ? kBoxRows : 0);
-    const int rb = max(1, min(rows_cap / m, (kRecCap / ng - 1) * kChunk));
-    const int rounds = (J1 - J0 + rb - 1) / rb;
+    const int rb = ng > 0 ? max(1, min(rows_cap / m, (kRecCap / ng - 1) * kChunk)) : 1;
+    const int rounds = ng > 0 ? (J1 - J0 + rb - 1) / rb : 0;
 
     if (tid == 0) {
         for (int st = 0; st < kStages; ++st) {
@@ -233,7 +295,7 @@ batch_kernel(Format f, const int2 *__restrict__ sets, const float *__restrict__ 
         else mbar_expect_tx(&full[st], hbytes);
         if (handle)
             for (int gi = 0; gi < ng; ++gi) {
-                const Group gg = f.groups[set.x + gi];
+                const Group gg = f.groups[gfirst + gi];
                 bulk_g2s(s_v0 + st * stage_val_bytes<BF16>() + size_t(gi) * bv,
                          static_cast<const unsigned char *>(f.vals) +
                              (size_t(gg.val_off) + size_t(g.cr0) * kSlots * kChunk) * kEsz,
@@ -323,12 +385,14 @@ batch_kernel(Format f, const int2 *__restrict__ sets, const float *__restrict__ 
         for (int u = 0; u < kQ; ++u) acc[p][u] = acc2[p][u] = make_float4(0.f, 0.f, 0.f, 0.f);
     const int rpt = (ng * kSlots + kConsumers * kRpw - 1) / (kConsumers * kRpw);
     uint32_t valid_mask = 0u;
+    // every row pass in use and no GRU split: all rows of a chunk at once
+    const bool all_rows = !kSplit && rpt == kRptMax;
     if (warp < kConsumers) {
 #pragma unroll
         for (int p = 0; p < kRptMax; ++p) {
             const int s = warp * kRpw + rr + p * kConsumers * kRpw;
             const int gi = s / kSlots;
-            if (p < rpt && gi < ng && (s % kSlots) < f.groups[set.x + gi].nrows) valid_mask |= 1u << p;
+            if (p < rpt && gi < ng && (s % kSlots) < f.groups[gfirst + gi].nrows) valid_mask |= 1u << p;
         }
         for (int r = 0; r < rounds && ok; ++r) {
             const int st = r % kStages;
@@ -344,6 +408,36 @@ batch_kernel(Format f, const int2 *__restrict__ sets, const float *__restrict__ 
                 // blocks of this chunk inside the round (all 8 except at the round's ends)
                 const int e_lo = max(0, g.jr0 - jc), e_hi = min(kChunk, g.jr1 - jc);
                 const bool whole = e_lo == 0 && e_hi == kChunk;
+                if constexpr (!kSplit) {
+                    if (all_rows) {
+                        // a row past the set (the last pass of an odd set) repeats a
+                        // row of its last group; its sums are never written
+                        int rec[kRptMax];
+#pragma unroll
+                        for (int p = 0; p < kRptMax; ++p) {
+                            const int s = warp * kRpw + rr + p * kConsumers * kRpw;
+                            const int gi = min(s / kSlots, ng - 1);
+                            rec[p] = (gi * g.nchr + lc) * kSlots + (s % kSlots);
+                        }
+                        // rows in sub-groups of kNpg, so that the values, offsets and
+                        // loads in flight of a sub-group fit in registers
+#pragma unroll
+                        for (int p0 = 0; p0 < kRptMax; p0 += kNpg) {
+#define DARB_ROWS(NIBV, WHOLEV)                                                                                 \
+    chunk_rows<BF16, NIBV, WHOLEV, kStacked, kNpg, kQ, LPR>(s_vals, s_offs, rec + p0, sx4, qd, g, jc, m, kBt / 4, \
+                                                           e_lo, e_hi, acc + p0)
+                            if (rw == 1) {
+                                if (whole) DARB_ROWS(true, true);
+                                else DARB_ROWS(true, false);
+                            } else {
+                                if (whole) DARB_ROWS(false, true);
+                                else DARB_ROWS(false, false);
+                            }
+#undef DARB_ROWS
+                        }
+                        continue;
+                    }
+                }
 #pragma unroll
                 for (int p = 0; p < kRptMax; ++p) {
                     if (valid_mask & (1u << p)) {
@@ -396,18 +490,20 @@ batch_kernel(Format f, const int2 *__restrict__ sets, const float *__restrict__ 
     }
     __syncthreads();
     if (ksc > 1) cluster.sync();
-    // rank q finishes rows [s0, s1) of the set for the whole tile
+    // this rank (index qsub of the ksub ranks sharing the set, cluster ranks
+    // qbase ..) finishes rows [s0, s1) of the set for the whole tile
+    const int ksub = item.ksub, qsub = item.qsub, qbase = q - qsub;
     const int R = ng * kSlots;
-    const int per = (R + ksc - 1) / ksc;
-    const int s0 = min(R, q * per), s1 = min(R, s0 + per);
+    const int per = (R + ksub - 1) / ksub;
+    const int s0 = min(R, qsub * per), s1 = min(R, s0 + per);
     for (int idx = tid; idx < (s1 - s0) * kBt * kParts; idx += kThreads) {
         const int s = s0 + idx / (kBt * kParts), pt = (idx / kBt) % kParts, t = idx % kBt;
         const int gi = s / kSlots, slot = s % kSlots;
-        if (b0 + t >= batch || slot >= f.groups[set.x + gi].nrows) continue;
+        if (b0 + t >= batch || slot >= f.groups[gfirst + gi].nrows) continue;
         float sum = 0.0f;   // ranks in a fixed order: deterministic
-        for (int r = 0; r < ksc; ++r)
-            sum += (ksc > 1 ? cluster.map_shared_rank(part, r) : part)[(s * kParts + pt) * kBt + t];
-        const int row = f.rowmap[(set.x + gi) * kSlots + slot];
+        for (int r = 0; r < ksub; ++r)
+            sum += (ksc > 1 ? cluster.map_shared_rank(part, qbase + r) : part)[(s * kParts + pt) * kBt + t];
+        const int row = f.rowmap[(gfirst + gi) * kSlots + slot];
         if constexpr (MODE == kModeY) Y[int64_t(row) * ldy + b0 + t] = sum;
         else (pt == 0 ? ra.gx : ra.gh)[int64_t(row) * ra.B + b0 + t] = sum;
     }
@@ -420,8 +516,8 @@ batch_kernel(Format f, const int2 *__restrict__ sets, const float *__restrict__ 
         __syncthreads();
         for (int s = s0 + tid; s < s1; s += kThreads) {
             const int gi = s / kSlots, slot = s % kSlots;
-            if (slot < f.groups[set.x + gi].nrows)
-                s_rows[atomicAdd(&s_nunits[1], 1)] = f.rowmap[(set.x + gi) * kSlots + slot];
+            if (slot < f.groups[gfirst + gi].nrows)
+                s_rows[atomicAdd(&s_nunits[1], 1)] = f.rowmap[(gfirst + gi) * kSlots + slot];
         }
         __syncthreads();
         const int nloc = s_nunits[1];
@@ -448,32 +544,31 @@ inline bool make_map(CUtensorMap *map, const float *A, int64_t ld, int64_t batch
 }
 
 // Grid shape of a plain product: row-set level l (sets of up to 2^l groups)
-// and cluster split k.
-// A CTA's work is proportional to 2^l / k plus a fixed cost (prologue,
-// reduction), about 0.2 in those units, and the launch takes
-// ceil(CTAs / resident CTAs) waves, so the cost is waves * (2^l / k + 0.2);
-// on a tie the shape with fewer waves wins, then the larger sets (each staged
-// activation row serves more rows).  Fitted to a sweep of every shape on
-// FC6/FC7 at batch 16-32, where sets of 4 groups split 8 ways (one wave) beat
-// sets of 2 groups split 8 ways (1.7 waves) by 25-35%.
+// and cluster size C = 2^c (the work table items[l][c]).
+// A CTA's work is at most item_work group-chunks, plus a fixed cost (prologue,
+// reduction) of about 0.2 x nch_max group-chunks, and the launch takes
+// ceil(CTAs / resident CTAs) waves, so the cost is
+// waves * (item_work / nch_max + 0.2); on a tie the shape with fewer waves
+// wins, then the larger sets (each staged activation row serves more rows).
 template <int LPR, int CPL>
-inline void grid_shape(const Format &f, int64_t tiles, int per_sm, int *level, unsigned *ksc) {
+inline void grid_shape(const Format &f, int64_t tiles, int per_sm, int *level, int *split) {
     const int64_t slots = int64_t(per_sm > 0 ? per_sm : 1) * sm_count();
     double best = 1e300;
     int64_t best_waves = 0;
     *level = 0;
-    *ksc = 1;
-    for (int l = 3; l >= 0; --l) {
-        if ((1 << l) > max_set_groups<LPR, CPL>() || f.nsets[l] <= 0) continue;
-        for (unsigned k = 8; k >= 1; k /= 2) {
-            const int64_t ctas = int64_t(f.nsets[l]) * tiles * k;
+    *split = 0;
+    for (int l = kWorkLevels - 1; l >= 0; --l) {
+        if ((1 << l) > max_set_groups<LPR, CPL>()) continue;
+        for (int c = kWorkSplits - 1; c >= 0; --c) {
+            if (f.nitems[l][c] <= 0) continue;
+            const int64_t ctas = int64_t(f.nitems[l][c]) * tiles;
             const int64_t waves = (ctas + slots - 1) / slots;
-            const double cost = double(waves) * (double(1 << l) / double(k) + 0.2);
+            const double cost = double(waves) * (double(f.item_work[l][c]) / double(f.nch_max) + 0.2);
             if (cost < best * (1 - 1e-9) || (cost <= best * (1 + 1e-9) && waves < best_waves)) {
                 best = cost;
                 best_waves = waves;
                 *level = l;
-                *ksc = k;
+                *split = c;
             }
         }
     }
@@ -484,16 +579,17 @@ inline void grid_shape(const Format &f, int64_t tiles, int per_sm, int *level, u
 // CTAs win there: the largest row sets that still give two CTAs per SM with a
 // split of 8, then the smallest split that reaches three CTAs per SM.
 template <int LPR, int CPL>
-inline void grid_shape_rnn(const Format &f, int64_t tiles, int *level, unsigned *ksc) {
+inline void grid_shape_rnn(const Format &f, int64_t tiles, int *level, int *split) {
     const int64_t want_min = 2 * int64_t(sm_count()), target = 3 * int64_t(sm_count());
+    const int cmax = kWorkSplits - 1;
     *level = 0;
-    for (int l = 3; l >= 0; --l) {
+    for (int l = kWorkLevels - 1; l >= 0; --l) {
         if ((1 << l) > max_set_groups<LPR, CPL>()) continue;
         *level = l;
-        if (int64_t(f.nsets[l]) * tiles * 8 >= want_min) break;
+        if (int64_t(f.nitems[l][cmax]) * tiles >= want_min) break;
     }
-    *ksc = 1;
-    while (*ksc < 8 && int64_t(f.nsets[*level]) * tiles * *ksc < target) *ksc *= 2;
+    *split = 0;
+    while (*split < cmax && int64_t(f.nitems[*level][*split]) * tiles < target) ++*split;
 }
 
 // CTAs of one batch_kernel instantiation resident per SM (shared memory is the limit).
@@ -529,13 +625,12 @@ cudaError_t launch(const Format &f, const float *X, int64_t ldx, int64_t batch, 
         use_tma = ok_x && ok_h ? 1 : 0;
     }
     const int64_t tiles = (batch + kBt - 1) / kBt;
-    int level;
-    unsigned ksc;
-    if constexpr (MODE == kModeY) grid_shape<LPR, CPL>(f, tiles, resident_per_sm<BF16, LPR, CPL, MODE>(), &level, &ksc);
-    else grid_shape_rnn<LPR, CPL>(f, tiles, &level, &ksc);
-    const dim3 grid(static_cast<unsigned>(f.nsets[level]) * ksc, static_cast<unsigned>(tiles));
-    return launch_ex(batch_kernel<BF16, LPR, CPL, MODE>, grid, dim3(kThreads), smem, stream, ksc, true, f,
-                     f.sets[level], X, ldx, batch, Y, ldy, xmap, hmap, ra, use_tma, early ? 1 : 0);
+    int level, split;
+    if constexpr (MODE == kModeY) grid_shape<LPR, CPL>(f, tiles, resident_per_sm<BF16, LPR, CPL, MODE>(), &level, &split);
+    else grid_shape_rnn<LPR, CPL>(f, tiles, &level, &split);
+    const dim3 grid(static_cast<unsigned>(f.nitems[level][split]), static_cast<unsigned>(tiles));
+    return launch_ex(batch_kernel<BF16, LPR, CPL, MODE>, grid, dim3(kThreads), smem, stream, 1u << split, true, f,
+                     f.items[level][split], X, ldx, batch, Y, ldy, xmap, hmap, ra, use_tma, early ? 1 : 0);
 }
 
 // Tile width by batch, within what one block of the largest m can stage.

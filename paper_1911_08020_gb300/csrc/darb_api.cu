@@ -29,15 +29,22 @@ struct darb_handle_s {
     std::vector<int32_t> rowmap, rowloc, row_m;
     std::vector<darb::EncTile> enc_tiles;   // every encoder tile, resolved
     int32_t max_tile = 0;                   // elements of the largest encoder tile (nb * m)
-    std::vector<int2> sets;        // row sets of up to 1, 2, 4, 8 groups, concatenated
-    int32_t nsets[4] = {0, 0, 0, 0};
+    std::vector<darb::WorkItem> items;   // CTA work tables of every (level, split), concatenated
+    int32_t item_first[darb::kWorkLevels][darb::kWorkSplits] = {};
+    int32_t nitems[darb::kWorkLevels][darb::kWorkSplits] = {};
+    int32_t item_work[darb::kWorkLevels][darb::kWorkSplits] = {};
+    std::vector<int64_t> set_prefix[darb::kWorkLevels];   // work of the row sets of items[l][0], prefix sums
+    std::vector<darb::SetGeo> xsets;                      // row sets of xres, both tables concatenated
+    int32_t xset_first[darb::kXresTables] = {}, nxsets[darb::kXresTables] = {};
+    std::vector<int64_t> xset_prefix[darb::kXresTables];
+    darb::SetGeo *d_xsets = nullptr;
     int64_t val_elems = 0, off_words = 0;
     // device memory: one allocation holding the layout, values and offsets
     void *dmem = nullptr;
     size_t dbytes = 0;
     Group *d_groups = nullptr;
     darb::EncTile *d_tiles = nullptr;
-    int2 *d_sets = nullptr;
+    darb::WorkItem *d_items = nullptr;
     int32_t *d_rowmap = nullptr, *d_rowloc = nullptr, *d_row_m = nullptr, *d_status = nullptr;
     void *d_vals = nullptr;
     uint32_t *d_offs = nullptr;
@@ -93,6 +100,8 @@ size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
 
 int64_t ceil_div(int64_t a, int64_t b) { return (a + b - 1) / b; }
 
+void build_work_tables(darb_handle_s *h);
+
 // Bin rows by block size (stable: ascending m, then ascending row) and cut
 // each bin into 32-row groups.
 void build_layout(darb_handle_s *h, const int32_t *m) {
@@ -141,22 +150,7 @@ void build_layout(darb_handle_s *h, const int32_t *m) {
     }
     h->val_elems = val;
     h->off_words = off;
-    // row sets: consecutive groups of one bin, at most 2^i per set
-    h->sets.clear();
-    for (int i = 0; i < 4; ++i) {
-        const int cap = 1 << i;
-        h->nsets[i] = 0;
-        size_t gbeg = 0;
-        while (gbeg < h->groups.size()) {
-            size_t gend = gbeg;
-            while (gend < h->groups.size() && h->groups[gend].m == h->groups[gbeg].m) ++gend;
-            for (size_t s = gbeg; s < gend; s += cap) {
-                h->sets.push_back(make_int2(static_cast<int>(s), static_cast<int>(std::min<size_t>(cap, gend - s))));
-                ++h->nsets[i];
-            }
-            gbeg = gend;
-        }
-    }
+    build_work_tables(h);
     h->enc_tiles.clear();
     h->max_tile = 0;
     for (int64_t r = 0; r < rows; ++r) {
@@ -181,12 +175,114 @@ void build_layout(darb_handle_s *h, const int32_t *m) {
     }
 }
 
+// The CTA work tables of batch_kernel (darb::WorkItem).  For row sets of up to
+// 2^l consecutive groups of one bin and clusters of C = 2^c CTAs, every set is
+// split over k = min(C, its chunks) CTAs, each multiplying a contiguous 1/k of
+// the chunks.  (Splitting the sets of heavy bins over more CTAs than those of
+// light bins, to give every CTA the same work, measured slower: a light set on
+// few CTAs becomes a long run of short rounds whose copies the two-stage ring
+// cannot hide.)  Sets are packed into clusters by descending k (powers of two,
+// so no set straddles two clusters) and the last cluster is filled with idle
+// ranks.
+void build_work_tables(darb_handle_s *h) {
+    h->items.clear();
+    for (int l = 0; l < darb::kWorkLevels; ++l) {
+        const int cap = 1 << l;
+        std::vector<int2> sets;   // (first group, groups)
+        size_t gbeg = 0;
+        while (gbeg < h->groups.size()) {
+            size_t gend = gbeg;
+            while (gend < h->groups.size() && h->groups[gend].m == h->groups[gbeg].m) ++gend;
+            for (size_t s = gbeg; s < gend; s += cap)
+                sets.push_back(make_int2(static_cast<int>(s), static_cast<int>(std::min<size_t>(cap, gend - s))));
+            gbeg = gend;
+        }
+        auto nch_of = [h](const int2 &s) {
+            return static_cast<int64_t>(ceil_div(h->groups[static_cast<size_t>(s.x)].n, kChunk));
+        };
+        for (int c = 0; c < darb::kWorkSplits; ++c) {
+            const int C = 1 << c;
+            std::vector<std::pair<int, int2>> ks;
+            for (const int2 &s : sets) {
+                int k = 1;
+                while (2 * k <= C && 2 * k <= nch_of(s)) k *= 2;
+                ks.push_back({k, s});
+            }
+            std::stable_sort(ks.begin(), ks.end(), [](const auto &a, const auto &b) { return a.first > b.first; });
+            h->item_first[l][c] = static_cast<int32_t>(h->items.size());
+            int64_t most = 0;
+            for (const auto &e : ks) {
+                const int k = e.first;
+                const int64_t nch = nch_of(e.second);
+                for (int q = 0; q < k; ++q) {
+                    darb::WorkItem it{};
+                    it.g0 = e.second.x;
+                    it.ng = static_cast<int16_t>(e.second.y);
+                    it.qsub = static_cast<int8_t>(q);
+                    it.ksub = static_cast<int8_t>(k);
+                    it.c0 = static_cast<int32_t>(nch * q / k);
+                    it.c1 = static_cast<int32_t>(nch * (q + 1) / k);
+                    most = std::max<int64_t>(most, int64_t(it.ng) * (it.c1 - it.c0));
+                    h->items.push_back(it);
+                }
+            }
+            while ((h->items.size() - h->item_first[l][c]) % C != 0) {
+                darb::WorkItem idle{};
+                idle.ksub = 1;
+                h->items.push_back(idle);
+            }
+            h->nitems[l][c] = static_cast<int32_t>(h->items.size()) - h->item_first[l][c];
+            h->item_work[l][c] = static_cast<int32_t>(std::min<int64_t>(most, INT32_MAX));
+        }
+        // the sets of items[l][0] (one CTA each, in set order) and their work
+        h->set_prefix[l].assign(1, 0);
+        for (const int2 &s : sets) h->set_prefix[l].push_back(h->set_prefix[l].back() + s.y * nch_of(s));
+    }
+    // Row sets of xres: each bin's groups in runs of G = the largest power of
+    // two <= 8 with G * nch(bin) <= base * nch(heaviest bin), so that every set
+    // is about `base` groups of the heaviest bin's work; bins in layout order
+    // (heaviest first).
+    h->xsets.clear();
+    const int64_t nch_max = h->groups.empty() ? 1 : ceil_div(h->groups.front().n, kChunk);
+    for (int i = 0; i < darb::kXresTables; ++i) {
+        const int64_t base = int64_t(2) << i;
+        h->xset_first[i] = static_cast<int32_t>(h->xsets.size());
+        h->xset_prefix[i].assign(1, 0);
+        size_t gbeg = 0;
+        while (gbeg < h->groups.size()) {
+            size_t gend = gbeg;
+            while (gend < h->groups.size() && h->groups[gend].m == h->groups[gbeg].m) ++gend;
+            const Group &g = h->groups[gbeg];
+            const int64_t nch = ceil_div(g.n, kChunk);
+            int G = 1;
+            while (2 * G <= 8 && 2 * G * nch <= base * nch_max) G *= 2;
+            for (size_t s = gbeg; s < gend; s += static_cast<size_t>(G)) {
+                darb::SetGeo sg{};
+                const size_t ng = std::min<size_t>(static_cast<size_t>(G), gend - s);
+                sg.g0 = static_cast<int32_t>(s);
+                sg.ng = static_cast<int32_t>(ng);
+                sg.m = g.m;
+                sg.n = g.n;
+                sg.nib = g.nib;
+                sg.nrows_last = h->groups[s + ng - 1].nrows;
+                sg.val_off = h->groups[s].val_off;
+                sg.off_off = h->groups[s].off_off;
+                h->xsets.push_back(sg);
+                h->xset_prefix[i].push_back(h->xset_prefix[i].back() + int64_t(ng) * nch);
+            }
+            gbeg = gend;
+        }
+        h->nxsets[i] = static_cast<int32_t>(h->xsets.size()) - h->xset_first[i];
+    }
+}
+
 darb_status_t alloc_device(darb_handle_s *h) {
     const size_t esz = h->wtype == DARB_BF16 ? 2 : 4;
     size_t o = 0;
     const size_t o_groups = o; o = align_up(o + h->groups.size() * sizeof(Group), 256);
     const size_t o_tiles = o;  o = align_up(o + h->enc_tiles.size() * sizeof(darb::EncTile), 256);
-    const size_t o_sets = o;   o = align_up(o + h->sets.size() * sizeof(int2), 256);
+    const size_t o_items = o;  o = align_up(o + h->items.size() * sizeof(darb::WorkItem), 256);
+    const size_t o_sgeo = o;   o = align_up(o + h->xsets.size() * sizeof(darb::SetGeo), 256);
     const size_t o_rowmap = o; o = align_up(o + h->rowmap.size() * 4, 256);
     const size_t o_rowloc = o; o = align_up(o + h->rowloc.size() * 4, 256);
     const size_t o_rowm = o;   o = align_up(o + h->row_m.size() * 4, 256);
@@ -201,7 +297,8 @@ darb_status_t alloc_device(darb_handle_s *h) {
     h->dbytes = o;
     h->d_groups = reinterpret_cast<Group *>(b + o_groups);
     h->d_tiles = reinterpret_cast<darb::EncTile *>(b + o_tiles);
-    h->d_sets = reinterpret_cast<int2 *>(b + o_sets);
+    h->d_items = reinterpret_cast<darb::WorkItem *>(b + o_items);
+    h->d_xsets = reinterpret_cast<darb::SetGeo *>(b + o_sgeo);
     h->d_rowmap = reinterpret_cast<int32_t *>(b + o_rowmap);
     h->d_rowloc = reinterpret_cast<int32_t *>(b + o_rowloc);
     h->d_row_m = reinterpret_cast<int32_t *>(b + o_rowm);
@@ -220,7 +317,10 @@ darb_status_t upload_layout(darb_handle_s *h, cudaStream_t stream) {
         e = cudaMemcpyAsync(h->d_tiles, h->enc_tiles.data(), h->enc_tiles.size() * sizeof(darb::EncTile),
                             cudaMemcpyHostToDevice, stream);
     if (e == cudaSuccess)
-        e = cudaMemcpyAsync(h->d_sets, h->sets.data(), h->sets.size() * sizeof(int2),
+        e = cudaMemcpyAsync(h->d_items, h->items.data(), h->items.size() * sizeof(darb::WorkItem),
+                            cudaMemcpyHostToDevice, stream);
+    if (e == cudaSuccess && !h->xsets.empty())
+        e = cudaMemcpyAsync(h->d_xsets, h->xsets.data(), h->xsets.size() * sizeof(darb::SetGeo),
                             cudaMemcpyHostToDevice, stream);
     if (e == cudaSuccess)
         e = cudaMemcpyAsync(h->d_rowmap, h->rowmap.data(), h->rowmap.size() * 4,
@@ -257,9 +357,19 @@ Format format_of(const darb_handle_s *h) {
     f.vals = h->d_vals;
     f.offs = h->d_offs;
     f.status = h->d_status;
-    for (int i = 0, o = 0; i < 4; o += h->nsets[i], ++i) {
-        f.sets[i] = h->d_sets + o;
-        f.nsets[i] = h->nsets[i];
+    for (int l = 0; l < darb::kWorkLevels; ++l)
+        for (int c = 0; c < darb::kWorkSplits; ++c) {
+            f.items[l][c] = h->d_items + h->item_first[l][c];
+            f.nitems[l][c] = h->nitems[l][c];
+            f.item_work[l][c] = h->item_work[l][c];
+        }
+    f.nch_max = h->groups.empty() ? 1 : static_cast<int32_t>(ceil_div(h->groups.front().n, kChunk));
+    for (int l = 0; l < darb::kWorkLevels; ++l) f.set_prefix[l] = h->set_prefix[l].data();
+    for (int i = 0; i < darb::kXresTables; ++i) {
+        f.xsets[i] = h->d_xsets + h->xset_first[i];
+        f.nxsets[i] = h->nxsets[i];
+        f.xset_prefix[i] = h->xset_prefix[i].data();
+        f.xsets_host[i] = h->xsets.data() + h->xset_first[i];
     }
     f.ngroups = static_cast<int32_t>(h->groups.size());
     f.bf16 = h->wtype == DARB_BF16 ? 1 : 0;

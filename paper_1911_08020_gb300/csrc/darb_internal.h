@@ -43,6 +43,39 @@ struct Group {
     int64_t off_off;  // uint32 word index of chunk 0 / slot 0 in the offset array
 };
 
+// One CTA's share of a product of batch_kernel: a row set (a run of up to 2^l
+// consecutive 32-row groups of one block-size bin) and the chunks of the set's
+// blocks that this CTA multiplies.  The ksub CTAs that share a set are
+// consecutive ranks of one thread-block cluster (qsub = this CTA's index among
+// them); they add their partial sums through distributed shared memory.
+struct WorkItem {
+    int32_t g0;      // first group of the set
+    int16_t ng;      // groups in the set; 0: an idle rank that only joins the cluster's barriers
+    int8_t qsub;     // this CTA's index among the CTAs that share the set
+    int8_t ksub;     // CTAs that share the set (consecutive ranks of one cluster)
+    int32_t c0, c1;  // chunks [c0, c1) of the set's blocks
+};
+constexpr int kWorkLevels = 4;   // row sets of up to 1, 2, 4, 8 groups
+
+// A row set of the resident-activation product (xres.cuh): a run of ng <= 8
+// consecutive groups of one bin, in one 48-byte record (no dependent lookups).
+// The groups of a bin have equal block counts, so group g0 + i starts i group
+// strides after the first: values at val_off + i * nch * 256, offsets at
+// off_off + i * nch * 32 * (nib ? 1 : 2) (nch = ceil(n / 8)); all groups are
+// full except possibly the last.
+struct __align__(16) SetGeo {
+    int32_t g0;           // first group
+    int32_t ng;           // groups (1..8)
+    int32_t m, n;         // block size and blocks per row
+    int32_t nib;          // 1: 4-bit offsets
+    int32_t nrows_last;   // rows in use of the last group
+    int64_t val_off;      // Group::val_off of the first group
+    int64_t off_off;      // Group::off_off of the first group
+    int64_t pad;
+};
+constexpr int kXresTables = 2;   // row-set tables of xres: 2 and 4 groups of the heaviest bin
+constexpr int kWorkSplits = 4;   // clusters of 1, 2, 4, 8 CTAs
+
 // Everything a kernel needs to read an encoded matrix.
 struct Format {
     const Group *groups;
@@ -52,10 +85,24 @@ struct Format {
     const void *vals;        // fp32 or bf16 bit patterns
     const uint32_t *offs;
     int32_t *status;         // sticky device status bits (NaN seen, wait timed out)
-    // row sets: runs of up to 1, 2, 4, 8 consecutive groups of one bin, as
-    // (first group, group count); sets[i] holds the sets of up to 2^i groups
-    const int2 *sets[4];
-    int32_t nsets[4];
+    // CTA work tables of batch_kernel: items[l][c] for row sets of up to 2^l
+    // groups and clusters of 2^c CTAs (nitems[l][c] entries, a multiple of 2^c;
+    // item_work[l][c] = the most group-chunks any one item multiplies)
+    const WorkItem *items[kWorkLevels][kWorkSplits];
+    int32_t nitems[kWorkLevels][kWorkSplits];
+    int32_t item_work[kWorkLevels][kWorkSplits];
+    int32_t nch_max;         // chunks of a row of the smallest block size
+    // HOST memory (never read by a kernel): for the row sets of level l in the
+    // order of items[l][0], set_prefix[l][s] = sum of the work (groups x
+    // chunks per row) of sets [0, s); nitems[l][0] + 1 entries
+    const int64_t *set_prefix[kWorkLevels];
+    // row sets of xres (SetGeo): table i sizes the sets of every bin to about
+    // the work of 2 << i groups of the heaviest bin (at most 8 groups); device
+    // records, and on the HOST the prefix sums of their work (group-chunks)
+    const SetGeo *xsets[kXresTables];
+    int32_t nxsets[kXresTables];
+    const int64_t *xset_prefix[kXresTables];
+    const SetGeo *xsets_host[kXresTables];   // HOST copies of xsets
     int32_t ngroups;
     int32_t bf16;            // value dtype: 0 fp32, 1 bf16
     int32_t m_max;           // largest block size of any row

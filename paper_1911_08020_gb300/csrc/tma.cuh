@@ -115,6 +115,51 @@ __device__ __forceinline__ void fence_proxy_async_global() {
     asm volatile("fence.proxy.async.global;" ::: "memory");
 }
 
+// Arrive on the mbarrier at the same shared-memory offset as `bar` in CTA
+// `rank` of this cluster, with the default semantics (release at CTA scope):
+// it orders this CTA's earlier accesses to its own shared memory (made by
+// other threads too, after a CTA barrier) before the arrival -- enough to
+// hand shared-memory data to another CTA, which reads it through distributed
+// shared memory -- without waiting for this CTA's global stores to drain, as
+// a release at cluster scope would.
+__device__ __forceinline__ void mbar_arrive_remote(uint64_t *bar, uint32_t rank) {
+    uint32_t remote;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(smem_addr(bar)), "r"(rank));
+    asm volatile("mbarrier.arrive.shared::cluster.b64 _, [%0];" ::"r"(remote) : "memory");
+}
+
+// mbar_wait with acquire at cluster scope, for phases completed by arrivals of
+// other CTAs of the cluster (mbar_arrive_remote); false after the time limit.
+// With `backoff` the thread sleeps between attempts (as mbar_wait), so that a
+// warp that waits long leaves the issue slots to the others.
+__device__ __forceinline__ bool mbar_wait_acq_cluster(uint64_t *bar, uint32_t parity, bool backoff = false) {
+    const uint32_t a = smem_addr(bar);
+    unsigned long long t0 = 0;
+    unsigned sleep_ns = 32;
+    while (true) {
+        uint32_t done;
+        asm volatile(
+            "{\n .reg .pred p;\n"
+            " mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2, %3;\n"
+            " selp.u32 %0, 1, 0, p;\n}\n"
+            : "=r"(done) : "r"(a), "r"(parity), "r"(10000u) : "memory");
+        if (done) return true;
+        const unsigned long long now = global_timer_ns();
+        if (t0 == 0) t0 = now;
+        else if (now - t0 > kWaitLimitNs) return false;
+        if (backoff) {
+            __nanosleep(sleep_ns);
+            if (sleep_ns < 512) sleep_ns <<= 1;
+        }
+    }
+}
+
+// Named barrier `id` (1..15) over `threads` threads of the CTA (a multiple of
+// 32; the warps that take part all call it with the same id and count).
+__device__ __forceinline__ void named_sync(uint32_t id, uint32_t threads) {
+    asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(threads) : "memory");
+}
+
 // Programmatic dependent launch: let the next kernel on the stream start its
 // prologue, and wait until the previous kernel's writes are visible.
 __device__ __forceinline__ void pdl_launch_dependents() {

@@ -1,0 +1,686 @@
+// xres.cuh -- Y = W_darb X for batch > 4 with each CTA's slice of the activation
+// tile resident in shared memory (Sec. 3.2, Fig. 6(b): block j of a row selects
+// activation row j*m + off).
+//
+// Why: the product multiplies every kept weight by one activation row of the
+// batch tile, and the rows a block can select are only its own m.  Split the
+// columns of W into C slices of S columns; a block belongs to the slice its
+// first column falls in, so a CTA that holds rows [q*S, (q+1)*S + m_max - 1)
+// of the tile can multiply every block of its slice, of every row, without
+// staging anything else.  A cluster of C CTAs (one per slice) therefore loads
+// the tile once and then streams only the kept values and packed offsets
+// (2.5 bytes per kept weight for bf16) through a ring of bulk copies.  The C
+// partial sums of a row meet in distributed shared memory.
+//
+// Layout of the work:
+//  * persistent clusters (as many as the GPU holds at once), one CTA per SM;
+//  * a unit = (batch tile of T columns, row set): a run of up to 8 groups of
+//    one block-size bin, sized so that every set has about the work of a
+//    fixed number of groups of the heaviest bin (the SetGeo tables of the
+//    handle); units in tile-major order; each cluster takes a contiguous run
+//    of units of about equal work, so it loads the tile of a run once or twice;
+//  * 16 consumer warps: T/4 lanes per row, each lane 4 columns (one 16-byte
+//    load per kept weight; a quarter-warp reads 64 or 128 contiguous bytes of
+//    one activation row); a thread owns 1 to 4 rows of the set and works on
+//    the same chunk of all of them at once, so their loads overlap;
+//  * one producer warp: bulk copies of the values and offsets of each round
+//    (a run of chunks of the set's groups) into a 6-stage ring with full /
+//    empty mbarriers, and tensor-map copies of the tile slice (rows past the
+//    matrix or columns past the batch arrive as zeros);
+//  * three reducer warps: when every CTA of the cluster has stored its partial
+//    sums of a set (each consumer warp, once its rows are stored, arrives on
+//    every CTA's "ready" barrier), they add, for this CTA's R/C rows, the C
+//    partial sums in rank order (deterministic), write Y, and each reducer
+//    warp arrives on every CTA's "freed" barrier; the consumers meanwhile
+//    multiply the next set, and store its partial sums only once every CTA's
+//    reducers have read the previous ones.  No CTA-wide barrier separates
+//    the sets.  (Every warp arrives once per set on each barrier, and issues
+//    its arrivals for set t + 1 on one barrier only after every CTA has got
+//    past set t on the other -- microseconds after every arrival for set t
+//    was issued.)
+//
+// Waits poll try_wait, which parks the warp in hardware until the phase
+// completes, without sleeping in between (a lane that slept past the phase
+// would hold up its warp).  Every wait is bounded; one that gives up records
+// DARB_ERR_TIMEOUT, the
+// warp skips the remaining work, the producer lets its own copies land
+// (bounded) and all warps meet at the final cluster barrier, so no CTA leaves
+// while another may still read its shared memory or arrive on its barriers.
+#pragma once
+
+#include "kernels_common.cuh"
+#include "launch.cuh"
+#include "tma.cuh"
+
+#include <cooperative_groups.h>
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
+#include <algorithm>
+#include <cstring>
+#include <type_traits>
+#include <vector>
+
+namespace darb {
+namespace xres {
+
+namespace cg = cooperative_groups;
+
+constexpr int kCWarps = 16;                    // consumer warps
+constexpr int kCThreads = kCWarps * 32;
+constexpr int kRWarps = 3;                     // reducer warps (20 warps in all: 96 registers a thread)
+constexpr int kRThreads = kRWarps * 32;
+constexpr int kProducerWarp = kCWarps;
+constexpr int kThreads = kCThreads + 32 + kRThreads;
+constexpr int kStages = 6;                     // rounds of values and offsets in the ring
+constexpr int kRecCap = 8;                     // (group, chunk) records per round
+constexpr int kMaxGroups = 8;                  // groups of a row set, at most
+constexpr int kMaxClusters = 160;
+constexpr int kUnitCost = 10;                  // fixed cost of a unit, in group-chunks
+constexpr size_t kSmemCap = 226 * 1024;        // dynamic shared memory, at most
+
+template <bool BF16>
+__host__ __device__ constexpr uint32_t rec_val_bytes() { return kSlots * kChunk * (BF16 ? 2 : 4); }
+constexpr uint32_t kRecOffBytes = kSlots * 8;  // room for 8-byte offset records
+template <bool BF16>
+__host__ __device__ constexpr uint32_t ring_val_bytes() { return kRecCap * rec_val_bytes<BF16>(); }
+template <bool BF16>
+__host__ __device__ constexpr uint32_t stage_bytes() { return ring_val_bytes<BF16>() + kRecCap * kRecOffBytes; }
+
+// Rows one pass of the consumers covers: T/4 lanes per row.
+template <int T>
+__host__ __device__ constexpr int pass_rows() { return kCWarps * 32 / (T / 4); }
+
+struct Plan {
+    int C;            // CTAs per cluster = column slices
+    int S;            // a slice's blocks start in columns [q*S, (q+1)*S)
+    int box_rows;     // activation rows per tensor-map box
+    int nboxes;       // boxes per slice
+    int table;        // row-set table (SetGeo) of the handle
+    int nsets;        // row sets of that table
+    uint32_t x_bytes; // bytes of the staged slice (nboxes * box_rows * T * 4)
+    uint32_t ring_off, part_off;   // offsets in dynamic shared memory
+    int2 range[kMaxClusters];      // units [x, y) of each cluster
+};
+
+// Barriers at the start of dynamic shared memory.
+struct Bars {
+    uint64_t full[kStages], empty[kStages];
+    uint64_t xfull, xfree;
+    uint64_t ready, freed;
+};
+static_assert(sizeof(Bars) <= 128, "the barriers fit in front of the slice");
+
+// A row set as the kernel keeps it in registers (constant indexing only).
+struct Set {
+    int g0, ng, m, n, nib, nrows_last;
+    long long val_off, off_off;
+};
+
+template <bool BF16, int T>
+__global__ void __launch_bounds__(kThreads, 1)
+xres_kernel(Format f, const float *__restrict__ X, int64_t batch, float *__restrict__ Y, int64_t ldy,
+            const __grid_constant__ CUtensorMap xmap, const __grid_constant__ Plan p) {
+    constexpr int kLpr = T / 4;             // lanes per row
+    constexpr int kRpw = 32 / kLpr;         // rows per warp and pass
+    constexpr int kPassRows = pass_rows<T>();
+    constexpr int kEsz = BF16 ? 2 : 4;
+    extern __shared__ __align__(128) unsigned char sm[];
+    Bars &bar = *reinterpret_cast<Bars *>(sm);
+    float *s_x = reinterpret_cast<float *>(sm + 128);
+    unsigned char *s_ring = sm + p.ring_off;
+    float *s_part = reinterpret_cast<float *>(sm + p.part_off);   // [8 * 32 rows][T]
+
+    pdl_launch_dependents();
+    cg::cluster_group cluster = cg::this_cluster();
+    const int C = p.C;
+    const int q = static_cast<int>(cluster.block_rank());
+    const int cl = static_cast<int>(blockIdx.x) / C;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int u_begin = p.range[cl].x, u_end = p.range[cl].y;
+    const SetGeo *sets = f.xsets[p.table];
+    const int kq0 = q * p.S;                // first activation row of the slice
+
+    if (tid == 0) {
+        for (int st = 0; st < kStages; ++st) {
+            mbar_init(&bar.full[st], 1);
+            mbar_init(&bar.empty[st], kCWarps);
+        }
+        mbar_init(&bar.xfull, 1);
+        mbar_init(&bar.xfree, kCWarps);
+        mbar_init(&bar.ready, kCWarps * C);   // every consumer warp of every CTA, once a set
+        mbar_init(&bar.freed, kRWarps * C);   // every reducer warp of every CTA, once a set
+        fence_mbar_init();
+    }
+    // every CTA's barriers exist before any CTA arrives on them remotely
+    cluster.sync();
+    pdl_wait_previous();   // X may come from the previous kernel, and Y may still be read by it
+
+    // A unit's row set, loaded one unit ahead so that its latency hides behind
+    // the current unit's work.
+    // (volatile loads: issued where they are written, a whole unit before use,
+    // instead of being moved down to it)
+    auto load_set = [&](int sidx) {
+        const int4 *src = reinterpret_cast<const int4 *>(sets + sidx);
+        int4 a, b, c;
+        asm volatile("ld.global.nc.v4.s32 {%0, %1, %2, %3}, [%4];" : "=r"(a.x), "=r"(a.y), "=r"(a.z), "=r"(a.w) : "l"(src));
+        asm volatile("ld.global.nc.v4.s32 {%0, %1, %2, %3}, [%4];" : "=r"(b.x), "=r"(b.y), "=r"(b.z), "=r"(b.w) : "l"(src + 1));
+        asm volatile("ld.global.nc.v4.s32 {%0, %1, %2, %3}, [%4];" : "=r"(c.x), "=r"(c.y), "=r"(c.z), "=r"(c.w) : "l"(src + 2));
+        Set s;
+        s.g0 = a.x; s.ng = a.y; s.m = a.z; s.n = a.w;
+        s.nib = b.x; s.nrows_last = b.y;
+        s.val_off = static_cast<long long>((static_cast<unsigned long long>(static_cast<unsigned>(b.w)) << 32) |
+                                           static_cast<unsigned>(b.z));
+        s.off_off = static_cast<long long>((static_cast<unsigned long long>(static_cast<unsigned>(c.y)) << 32) |
+                                           static_cast<unsigned>(c.x));
+        return s;
+    };
+    // This CTA's share of a unit: blocks [j0, j1), chunks [c0, c0 + nch), in rounds of cpr chunks.
+    struct Unit {
+        int tile, j0, j1, c0, nch, cpr, rounds;
+    };
+    // Unit u = tile * nsets + sidx; the running position (no division per unit).
+    struct Cursor {
+        int tile, sidx;
+    };
+    auto cursor_at = [&](int u) {
+        Cursor c;
+        c.tile = u / p.nsets;
+        c.sidx = u - c.tile * p.nsets;
+        return c;
+    };
+    auto advance = [&](Cursor &c) {
+        if (++c.sidx == p.nsets) {
+            c.sidx = 0;
+            ++c.tile;
+        }
+    };
+    // The first blocks of this slice in a row of block size m, ceil(q*S / m) and
+    // ceil((q+1)*S / m), recomputed only when m changes (the sets of a bin are
+    // consecutive, so a CTA divides a few times per launch).
+    int geo_m = -1, geo_ja = 0, geo_jb = 0;
+    auto unit_geo = [&](int tile, const Set &s) {
+        Unit g;
+        g.tile = tile;
+        if (s.m != geo_m) {
+            const unsigned lo = static_cast<unsigned>(q) * static_cast<unsigned>(p.S), hi = lo + static_cast<unsigned>(p.S);
+            const unsigned mu = static_cast<unsigned>(s.m);
+            geo_m = s.m;
+            geo_ja = static_cast<int>((lo + mu - 1) / mu);
+            geo_jb = static_cast<int>((hi + mu - 1) / mu);
+        }
+        g.j0 = geo_ja < s.n ? geo_ja : s.n;
+        g.j1 = geo_jb < s.n ? geo_jb : s.n;
+        g.c0 = g.j0 / kChunk;
+        g.nch = g.j1 > g.j0 ? (g.j1 + kChunk - 1) / kChunk - g.c0 : 0;
+        g.cpr = max(1, kRecCap / max(1, s.ng));
+        g.rounds = (g.nch + g.cpr - 1) / g.cpr;
+        return g;
+    };
+
+    if (warp == kProducerWarp) {
+        // ------------------------------------------------------------ producer
+        bool ok = true;
+        int rc = 0;           // rounds issued
+        int xloads = 0;       // slices loaded
+        int cur_tile = -1;
+        Cursor cu = cursor_at(u_begin), cn = cu;
+        advance(cn);
+        Set s_next = u_begin < u_end ? load_set(cu.sidx) : Set{};
+        for (int u = u_begin; u < u_end && ok; ++u, cu = cn, advance(cn)) {
+            const Set s = s_next;
+            if (u + 1 < u_end) s_next = load_set(cn.sidx);
+            const Unit g = unit_geo(cu.tile, s);
+            if (g.tile != cur_tile) {
+                // the consumers are done with the previous slice
+                if (xloads > 0) ok = mbar_wait(&bar.xfree, (xloads - 1) & 1, false);
+                ok = __shfl_sync(0xFFFFFFFFu, ok ? 1 : 0, 0) != 0;
+                if (!ok) break;
+                if (lane == 0) {
+                    fence_proxy_async_smem();
+                    mbar_arrive_expect_tx(&bar.xfull, p.x_bytes);
+                    for (int i = 0; i < p.nboxes; ++i)
+                        tensor2d_g2s(s_x + size_t(i) * p.box_rows * T, &xmap, g.tile * T, kq0 + i * p.box_rows,
+                                     &bar.xfull);
+                }
+                ++xloads;
+                cur_tile = g.tile;
+            }
+            const int rw = s.nib ? 1 : 2;
+            const int64_t gnch = (s.n + kChunk - 1) / kChunk;   // chunks of a group
+            for (int r = 0; r < g.rounds; ++r, ++rc) {
+                const int st = rc % kStages;
+                if (rc >= kStages) ok = mbar_wait(&bar.empty[st], ((rc / kStages) - 1) & 1, false);
+                ok = __shfl_sync(0xFFFFFFFFu, ok ? 1 : 0, 0) != 0;
+                if (!ok) break;
+                if (lane == 0) {
+                    const int cr0 = g.c0 + r * g.cpr, nchr = min(g.cpr, g.nch - r * g.cpr);
+                    const uint32_t bv = uint32_t(nchr) * kSlots * kChunk * kEsz;
+                    const uint32_t bo = uint32_t(nchr) * kSlots * rw * 4;
+                    unsigned char *sv = s_ring + size_t(st) * stage_bytes<BF16>();
+                    unsigned char *so = sv + ring_val_bytes<BF16>();
+                    fence_proxy_async_smem();
+                    mbar_arrive_expect_tx(&bar.full[st], uint32_t(s.ng) * (bv + bo));
+                    for (int gi = 0; gi < s.ng; ++gi) {
+                        const int64_t vo = s.val_off + (gi * gnch + cr0) * (kSlots * kChunk);
+                        const int64_t oo = s.off_off + (gi * gnch + cr0) * (kSlots * rw);
+                        bulk_g2s(sv + size_t(gi) * bv, static_cast<const unsigned char *>(f.vals) + vo * kEsz, bv,
+                                 &bar.full[st]);
+                        bulk_g2s(so + size_t(gi) * bo, f.offs + oo, bo, &bar.full[st]);
+                    }
+                }
+            }
+        }
+        if (!ok && lane == 0) atomicOr(f.status, kStatusTimeout);
+        // the copies this CTA started have landed before it can leave
+        if (lane == 0) {
+            for (int k = 1; k <= kStages && k <= rc; ++k) {
+                const int last = rc - k;
+                mbar_wait(&bar.full[last % kStages], (last / kStages) & 1);
+            }
+            if (xloads > 0) mbar_wait(&bar.xfull, (xloads - 1) & 1);
+        }
+    } else if (warp > kProducerWarp) {
+        // ------------------------------------------------------------ reducers
+        const int rt = tid - (kCThreads + 32);   // 0 .. kRThreads-1
+        bool ok = true;
+        Cursor cu = cursor_at(u_begin), cn = cu;
+        advance(cn);
+        Set s_next = u_begin < u_end ? load_set(cu.sidx) : Set{};
+        for (int u = u_begin, t = 0; u < u_end; ++u, ++t, cu = cn, advance(cn)) {
+            const Set s = s_next;
+            if (u + 1 < u_end) s_next = load_set(cn.sidx);
+            if (ok) ok = mbar_wait_acq_cluster(&bar.ready, t & 1);
+            if (ok) {
+                const int64_t tile = cu.tile;
+                const int rows_per = s.ng * kSlots / C;   // C divides 32
+                for (int i = rt; i < rows_per * (T / 4); i += kRThreads) {
+                    const int row = q * rows_per + i / (T / 4), c4 = i % (T / 4);
+                    const int gg = row / kSlots, sl = row % kSlots;
+                    if (gg == s.ng - 1 && sl >= s.nrows_last) continue;
+                    const int idx = row * (T / 4) + c4;
+                    // ranks in a fixed order (deterministic), four loads in flight at a time
+                    float4 sum = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+                    for (int h = 0; h < 8; h += 4) {
+                        float4 pv[4];
+#pragma unroll
+                        for (int r = 0; r < 4; ++r)
+                            if (h + r < C)
+                                pv[r] = reinterpret_cast<const float4 *>(cluster.map_shared_rank(s_part, h + r))[idx];
+#pragma unroll
+                        for (int r = 0; r < 4; ++r)
+                            if (h + r < C) {
+                                if (h + r == 0) {
+                                    sum = pv[r];
+                                } else {
+                                    sum.x += pv[r].x;
+                                    sum.y += pv[r].y;
+                                    sum.z += pv[r].z;
+                                    sum.w += pv[r].w;
+                                }
+                            }
+                    }
+                    float *yr = Y + int64_t(f.rowmap[(s.g0 + gg) * kSlots + sl]) * ldy;
+                    const int64_t b0 = tile * T + c4 * 4;
+                    if (b0 < batch) yr[b0] = sum.x;
+                    if (b0 + 1 < batch) yr[b0 + 1] = sum.y;
+                    if (b0 + 2 < batch) yr[b0 + 2] = sum.z;
+                    if (b0 + 3 < batch) yr[b0 + 3] = sum.w;
+                }
+            }
+            // this warp is done reading the partial sums of every CTA: tell them all
+            __syncwarp();
+            if (lane < C) mbar_arrive_remote(&bar.freed, static_cast<uint32_t>((q + lane) % C));   // one lane per CTA
+        }
+        if (!ok && lane == 0) atomicOr(f.status, kStatusTimeout);
+    } else {
+        // ------------------------------------------------------------ consumers
+        const int qd = lane % kLpr;                 // float4 of the tile this lane owns
+        const int rs = warp * kRpw + lane / kLpr;   // row of the set in pass 0
+        bool ok = true;
+        int rc = 0, xloads = 0, cur_tile = -1;
+        Cursor cu = cursor_at(u_begin), cn = cu;
+        advance(cn);
+        Set s_next = u_begin < u_end ? load_set(cu.sidx) : Set{};
+        // this lane's 16 bytes of row 0 of the slice
+        const unsigned char *xl = reinterpret_cast<const unsigned char *>(s_x) + qd * 16;
+        constexpr int kRowShift = T == 32 ? 7 : 6;   // bytes of a staged activation row, log2
+        // one unit with NP row passes and 4-bit (NIB) or 8-bit offsets:
+        // multiply, then store the partial sums once every CTA's reducers
+        // have read the previous set's (t: sets stored)
+        auto unit = [&](auto npc, auto nibc, const Set &s, const Unit &g, int t) {
+            constexpr int NP = decltype(npc)::value;
+            constexpr bool NIB = decltype(nibc)::value;
+            float4 acc[NP];
+#pragma unroll
+            for (int pp = 0; pp < NP; ++pp) acc[pp] = make_float4(0.f, 0.f, 0.f, 0.f);
+            float4 acc2 = make_float4(0.f, 0.f, 0.f, 0.f);   // odd chunks of a chunk pair (NP == 1)
+            // a row past the set (the last pass of a set with fewer groups) repeats a
+            // row of its last group; its sums are stored but never read
+            int gip[NP], slotp[NP];
+#pragma unroll
+            for (int pp = 0; pp < NP; ++pp) {
+                const int row = rs + pp * kPassRows;
+                gip[pp] = min(row / kSlots, s.ng - 1);
+                slotp[pp] = row % kSlots;
+            }
+            const int mrow = s.m << kRowShift;   // bytes between the first rows of consecutive blocks
+            for (int r = 0; r < g.rounds; ++r, ++rc) {
+                const int st = rc % kStages;
+                if (ok) ok = mbar_wait(&bar.full[st], (rc / kStages) & 1, false);
+                ok = __shfl_sync(0xFFFFFFFFu, ok ? 1 : 0, 0) != 0;
+                if (ok) {
+                    const int cr0 = g.c0 + r * g.cpr, nchr = min(g.cpr, g.nch - r * g.cpr);
+                    const unsigned char *sv = s_ring + size_t(st) * stage_bytes<BF16>();
+                    const uint32_t *so = reinterpret_cast<const uint32_t *>(sv + ring_val_bytes<BF16>());
+                    int lc = 0;
+                    if constexpr (NP == 1) {
+                        // one row a thread: two whole chunks at a time, into two
+                        // accumulators, so that 16 gathers are in flight and the
+                        // records of both chunks load together
+                        const int slot0 = slotp[0], gi0 = gip[0];
+                        for (; lc + 1 < nchr; lc += 2) {
+                            const int jc = (cr0 + lc) * kChunk;
+                            if (jc < g.j0 || jc + 2 * kChunk > g.j1) break;   // not two whole chunks
+                            const int rec0 = (gi0 * nchr + lc) * kSlots + slot0, rec1 = rec0 + kSlots;
+                            uint32_t va[BF16 ? 4 : 8], vb[BF16 ? 4 : 8];
+                            uint2 oa, ob;
+                            {
+                                const uint4 *pa = reinterpret_cast<const uint4 *>(sv) + rec0 * (BF16 ? 1 : 2);
+                                const uint4 *pb = reinterpret_cast<const uint4 *>(sv) + rec1 * (BF16 ? 1 : 2);
+                                const uint4 a0 = pa[0], b0 = pb[0];
+                                va[0] = a0.x; va[1] = a0.y; va[2] = a0.z; va[3] = a0.w;
+                                vb[0] = b0.x; vb[1] = b0.y; vb[2] = b0.z; vb[3] = b0.w;
+                                if constexpr (!BF16) {
+                                    const uint4 a1 = pa[1], b1 = pb[1];
+                                    va[4] = a1.x; va[5] = a1.y; va[6] = a1.z; va[7] = a1.w;
+                                    vb[4] = b1.x; vb[5] = b1.y; vb[6] = b1.z; vb[7] = b1.w;
+                                }
+                                if constexpr (NIB) {
+                                    oa = make_uint2(so[rec0], 0u);
+                                    ob = make_uint2(so[rec1], 0u);
+                                } else {
+                                    oa = reinterpret_cast<const uint2 *>(so)[rec0];
+                                    ob = reinterpret_cast<const uint2 *>(so)[rec1];
+                                }
+                            }
+                            const int xa = (jc * s.m - kq0) << kRowShift, xbb = xa + (s.m << (kRowShift + 3));
+                            float4 &a = acc[0];
+                            float4 &b = acc2;
+#pragma unroll
+                            for (int e = 0; e < kChunk; ++e) {
+                                int offa, offb;
+                                if constexpr (NIB) {
+                                    offa = int((oa.x >> (4 * e)) & 15u);
+                                    offb = int((ob.x >> (4 * e)) & 15u);
+                                } else {
+                                    offa = int(((e < 4 ? oa.x : oa.y) >> (8 * (e & 3))) & 255u);
+                                    offb = int(((e < 4 ? ob.x : ob.y) >> (8 * (e & 3))) & 255u);
+                                }
+                                float wa, wb;
+                                if constexpr (BF16) {
+                                    wa = __uint_as_float((e & 1) ? (va[e >> 1] & 0xFFFF0000u) : (va[e >> 1] << 16));
+                                    wb = __uint_as_float((e & 1) ? (vb[e >> 1] & 0xFFFF0000u) : (vb[e >> 1] << 16));
+                                } else {
+                                    wa = __uint_as_float(va[e]);
+                                    wb = __uint_as_float(vb[e]);
+                                }
+                                const float4 x0 = *reinterpret_cast<const float4 *>(xl + (xa + e * mrow + (offa << kRowShift)));
+                                const float4 x1 = *reinterpret_cast<const float4 *>(xl + (xbb + e * mrow + (offb << kRowShift)));
+                                a.x = fmaf(wa, x0.x, a.x);
+                                a.y = fmaf(wa, x0.y, a.y);
+                                a.z = fmaf(wa, x0.z, a.z);
+                                a.w = fmaf(wa, x0.w, a.w);
+                                b.x = fmaf(wb, x1.x, b.x);
+                                b.y = fmaf(wb, x1.y, b.y);
+                                b.z = fmaf(wb, x1.z, b.z);
+                                b.w = fmaf(wb, x1.w, b.w);
+                            }
+                        }
+                    }
+                    for (; lc < nchr; ++lc) {
+                        const int jc = (cr0 + lc) * kChunk;
+                        const int e_lo = max(0, g.j0 - jc), e_hi = min(kChunk, g.j1 - jc);
+                        // byte offset of the slice row selected by block jc + e:
+                        // ((jc + e) * m + off - kq0) << kRowShift (xb is negative for a first
+                        // chunk whose leading blocks belong to the previous slice; those
+                        // blocks are never read)
+                        const int xb = (jc * s.m - kq0) << kRowShift;
+                        // rows in sub-groups of kSub, so that their values, offsets and
+                        // loads in flight fit in registers
+                        constexpr int kSub = NP < 2 ? NP : 2;
+#pragma unroll
+                        for (int p0 = 0; p0 < NP; p0 += kSub) {
+                            uint32_t vw[kSub][BF16 ? 4 : 8];
+                            uint2 ow[kSub];
+#pragma unroll
+                            for (int k = 0; k < kSub; ++k) {
+                                const int rec = (gip[p0 + k] * nchr + lc) * kSlots + slotp[p0 + k];
+                                const uint4 *pv = reinterpret_cast<const uint4 *>(sv) + rec * (BF16 ? 1 : 2);
+                                const uint4 w0 = pv[0];
+                                vw[k][0] = w0.x; vw[k][1] = w0.y; vw[k][2] = w0.z; vw[k][3] = w0.w;
+                                if constexpr (!BF16) {
+                                    const uint4 w1 = pv[1];
+                                    vw[k][4] = w1.x; vw[k][5] = w1.y; vw[k][6] = w1.z; vw[k][7] = w1.w;
+                                }
+                                if constexpr (NIB) ow[k] = make_uint2(so[rec], 0u);
+                                else ow[k] = reinterpret_cast<const uint2 *>(so)[rec];
+                            }
+                            // block e of row p0 + k: its kept value times its selected activation row
+                            auto block = [&](int e, int k) {
+                                int off;
+                                if constexpr (NIB) off = int((ow[k].x >> (4 * e)) & 15u);
+                                else off = int(((e < 4 ? ow[k].x : ow[k].y) >> (8 * (e & 3))) & 255u);
+                                float v;
+                                if constexpr (BF16)
+                                    v = __uint_as_float((e & 1) ? (vw[k][e >> 1] & 0xFFFF0000u) : (vw[k][e >> 1] << 16));
+                                else
+                                    v = __uint_as_float(vw[k][e]);
+                                const float4 xv =
+                                    *reinterpret_cast<const float4 *>(xl + (xb + e * mrow + (off << kRowShift)));
+                                float4 &a = acc[p0 + k];
+                                a.x = fmaf(v, xv.x, a.x);
+                                a.y = fmaf(v, xv.y, a.y);
+                                a.z = fmaf(v, xv.z, a.z);
+                                a.w = fmaf(v, xv.w, a.w);
+                            };
+                            if (e_lo == 0 && e_hi == kChunk) {
+                                // a whole chunk: one straight run, every load can be issued early
+#pragma unroll
+                                for (int e = 0; e < kChunk; ++e)
+#pragma unroll
+                                    for (int k = 0; k < kSub; ++k) block(e, k);
+                            } else {
+#pragma unroll
+                                for (int e = 0; e < kChunk; ++e)
+                                    if (e >= e_lo && e < e_hi)
+#pragma unroll
+                                        for (int k = 0; k < kSub; ++k) block(e, k);
+                            }
+                        }
+                    }
+                }
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&bar.empty[st]);
+            }
+            if constexpr (NP == 1) {   // the two chunk streams, in a fixed order
+                acc[0].x += acc2.x;
+                acc[0].y += acc2.y;
+                acc[0].z += acc2.z;
+                acc[0].w += acc2.w;
+            }
+            if (t >= 1 && ok) ok = mbar_wait_acq_cluster(&bar.freed, (t - 1) & 1);
+#pragma unroll
+            for (int pp = 0; pp < NP; ++pp)
+                reinterpret_cast<float4 *>(s_part)[(rs + pp * kPassRows) * kLpr + qd] = acc[pp];
+        };
+        int t = 0;   // sets stored
+        for (int u = u_begin; u < u_end; ++u, ++t, cu = cn, advance(cn)) {
+            const Set s = s_next;
+            if (u + 1 < u_end) s_next = load_set(cn.sidx);
+            const Unit g = unit_geo(cu.tile, s);
+            if (g.tile != cur_tile) {
+                if (xloads > 0) {   // done with the previous slice
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(&bar.xfree);
+                }
+                if (ok) ok = mbar_wait(&bar.xfull, xloads & 1, false);
+                ok = __shfl_sync(0xFFFFFFFFu, ok ? 1 : 0, 0) != 0;
+                ++xloads;
+                cur_tile = g.tile;
+            }
+            const int np = (s.ng * kSlots + kPassRows - 1) / kPassRows;
+            using N1 = std::integral_constant<int, 1>;
+            using N2 = std::integral_constant<int, 2>;
+            using N4 = std::integral_constant<int, 4>;
+            using Nib = std::true_type;
+            using Byte = std::false_type;
+            if (np <= 1) {
+                if (s.nib) unit(N1{}, Nib{}, s, g, t);
+                else unit(N1{}, Byte{}, s, g, t);
+            } else if (np == 2) {
+                if (s.nib) unit(N2{}, Nib{}, s, g, t);
+                else unit(N2{}, Byte{}, s, g, t);
+            } else if constexpr (4 * kPassRows <= kMaxGroups * kSlots) {
+                if (s.nib) unit(N4{}, Nib{}, s, g, t);
+                else unit(N4{}, Byte{}, s, g, t);
+            }
+            // this warp's partial sums are stored: tell every CTA's reducers
+            __syncwarp();
+            if (lane < C) mbar_arrive_remote(&bar.ready, static_cast<uint32_t>((q + lane) % C));   // one lane per CTA
+        }
+        // every CTA's reducers have read this CTA's last partial sums
+        if (t >= 1 && ok) ok = mbar_wait_acq_cluster(&bar.freed, (t - 1) & 1);
+        if (xloads > 0) {
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&bar.xfree);
+        }
+        if (!ok && lane == 0) atomicOr(f.status, kStatusTimeout);
+    }
+    cluster.sync();   // no CTA leaves while another may still read its shared memory
+}
+
+
+// Clusters of C CTAs of this kernel resident at once with `smem` bytes each.
+template <bool BF16, int T>
+inline int max_clusters(int C, uint32_t smem) {
+    const auto fn = xres_kernel<BF16, T>;
+    return static_cast<int>(per_device(reinterpret_cast<const void *>(fn), (long long)C << 32 | smem, [&]() -> long long {
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3(static_cast<unsigned>(C) * 64);
+        cfg.blockDim = dim3(kThreads);
+        cfg.dynamicSmemBytes = smem;
+        cudaLaunchAttribute at[1];
+        at[0].id = cudaLaunchAttributeClusterDimension;
+        at[0].val.clusterDim.x = static_cast<unsigned>(C);
+        at[0].val.clusterDim.y = 1;
+        at[0].val.clusterDim.z = 1;
+        cfg.attrs = at;
+        cfg.numAttrs = 1;
+        int n = 0;
+        if (cudaOccupancyMaxActiveClusters(&n, fn, &cfg) != cudaSuccess) {
+            cudaGetLastError();
+            n = 0;
+        }
+        return n;
+    }));
+}
+
+// The product on this kernel, or cudaErrorNotSupported when the call does not
+// fit it (the slice of the tile does not fit in shared memory even split 8
+// ways, or X cannot be described by a tensor map).
+template <bool BF16, int T>
+cudaError_t launch(const Format &f, const float *X, int64_t ldx, int64_t batch, float *Y, int64_t ldy, bool early,
+                   cudaStream_t stream) {
+    (void)early;
+    const int table = T == 32 ? 0 : 1;   // sets of about 2 (T = 32) or 4 (T = 16) heaviest groups
+    const int nsets = f.nxsets[table];
+    const int64_t tiles = (batch + T - 1) / T;
+    const int64_t units = tiles * nsets;
+    if (nsets <= 0 || units > (int64_t(1) << 30) || f.xset_prefix[table] == nullptr) return cudaErrorNotSupported;
+    if (reinterpret_cast<uintptr_t>(X) % 16 != 0 || (ldx * 4) % 16 != 0) return cudaErrorNotSupported;
+    PFN_cuTensorMapEncodeTiled_v12000 enc = tensor_map_encoder();
+    if (enc == nullptr) return cudaErrorNotSupported;
+    Plan p{};
+    uint32_t smem = 0;
+    // smallest split whose slice fits beside the ring and the partial sums of
+    // the largest set (8 groups)
+    for (int C = 1;; C *= 2) {
+        if (C > 8) return cudaErrorNotSupported;
+        const int64_t S = (f.cols + C - 1) / C;
+        const int64_t rows = std::min<int64_t>(f.cols, S + f.m_max - 1);
+        const int nboxes = static_cast<int>((rows + 255) / 256);
+        int box_rows = static_cast<int>((rows + nboxes - 1) / nboxes);
+        if (T == 16) box_rows = (box_rows + 1) & ~1;   // every box lands on a 128-byte boundary
+        const uint64_t x_bytes = uint64_t(nboxes) * box_rows * T * 4;
+        const uint64_t ring_off = 128 + x_bytes;
+        const uint64_t part_off = ring_off + uint64_t(kStages) * stage_bytes<BF16>();
+        const uint64_t total = part_off + uint64_t(kMaxGroups) * kSlots * T * 4;
+        if (total <= kSmemCap) {
+            p.C = C;
+            p.S = static_cast<int>(S);
+            p.box_rows = box_rows;
+            p.nboxes = nboxes;
+            p.x_bytes = static_cast<uint32_t>(x_bytes);
+            p.ring_off = static_cast<uint32_t>(ring_off);
+            p.part_off = static_cast<uint32_t>(part_off);
+            smem = static_cast<uint32_t>(total);
+            break;
+        }
+    }
+    p.table = table;
+    p.nsets = nsets;
+    const cudaError_t attr = allow_smem(xres_kernel<BF16, T>, kSmemCap);
+    if (attr != cudaSuccess) return attr;
+    const int ncl = static_cast<int>(
+        std::min<int64_t>({int64_t(max_clusters<BF16, T>(p.C, smem)), int64_t(kMaxClusters), units}));
+    if (ncl <= 0) return cudaErrorNotSupported;
+    // contiguous runs of units of about equal time: cluster c starts at the
+    // first unit whose cumulative cost reaches c / ncl of the total.  The ranks
+    // of a cluster go through a unit together, so a unit costs what its
+    // busiest rank streams -- its set's groups times the most chunks any
+    // slice's blocks touch -- plus a fixed cost per unit (the hand-off of its
+    // partial sums and the start of its rounds: about kUnitCost group-chunks
+    // of multiplying, measured on FC6/FC7).
+    thread_local std::vector<int64_t> cost;   // host; reused across calls
+    const SetGeo *hs = f.xsets_host[table];
+    cost.assign(static_cast<size_t>(nsets) + 1, 0);
+    for (int s = 0; s < nsets; ++s) {
+        int64_t most = 0;
+        for (int qq = 0; qq < p.C; ++qq) {
+            const int64_t lo = int64_t(qq) * p.S, hi = lo + p.S;
+            const int64_t j0 = std::min<int64_t>(hs[s].n, (lo + hs[s].m - 1) / hs[s].m);
+            const int64_t j1 = std::min<int64_t>(hs[s].n, (hi + hs[s].m - 1) / hs[s].m);
+            if (j1 > j0) most = std::max<int64_t>(most, (j1 + kChunk - 1) / kChunk - j0 / kChunk);
+        }
+        cost[static_cast<size_t>(s) + 1] = cost[static_cast<size_t>(s)] + hs[s].ng * most + kUnitCost;
+    }
+    const int64_t *pre = cost.data();
+    const int64_t wt = pre[nsets];
+    const int64_t wtot = wt * tiles;
+    auto first_unit = [&](int c) -> int64_t {
+        if (c >= ncl) return units;
+        const int64_t target = (wtot * c + ncl - 1) / ncl;   // first unit with start >= target
+        const int64_t tile = target / wt, rem = target % wt;
+        const int64_t s = std::lower_bound(pre, pre + nsets, rem) - pre;
+        return tile * nsets + s;
+    };
+    for (int c = 0; c < ncl; ++c)
+        p.range[c] = make_int2(static_cast<int>(first_unit(c)), static_cast<int>(first_unit(c + 1)));
+    CUtensorMap xmap;
+    std::memset(&xmap, 0, sizeof xmap);
+    const cuuint64_t dims[2] = {cuuint64_t(batch), cuuint64_t(f.cols)};
+    const cuuint64_t strides[1] = {cuuint64_t(ldx) * 4};
+    const cuuint32_t box[2] = {cuuint32_t(T), cuuint32_t(p.box_rows)};
+    const cuuint32_t estr[2] = {1, 1};
+    if (enc(&xmap, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, const_cast<float *>(X), dims, strides, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+        return cudaErrorNotSupported;
+    return launch_ex(xres_kernel<BF16, T>, dim3(static_cast<unsigned>(ncl * p.C)), dim3(kThreads), smem, stream,
+                     static_cast<unsigned>(p.C), true, f, X, batch, Y, ldy, xmap, p);
+}
+
+}  // namespace xres
+}  // namespace darb
