@@ -47,8 +47,6 @@ def parse_args():
     p.add_argument("--no-cpu", action="store_true")
     p.add_argument("--no-rnn", action="store_true")
     p.add_argument("--no-baselines", action="store_true", help="skip the cuSPARSE comparison section")
-    p.add_argument("--cpu-seconds", type=float, default=30.0,
-                   help="CPU time budget of the oracle arm (--impl reference) over all its steps")
     p.add_argument("--calls", default="",
                    help="comma list restricting the step to some calls, e.g. fc6_spmm_b256 (profiling)")
     return p.parse_args()
@@ -79,18 +77,22 @@ _COMMON_SOURCES = ("darb_internal.h", "launch.cuh", "tma.cuh", "spmm.cu")
 _CALL_SOURCES = {
     "encode": ("encode.cu",),
     "b1": ("gemv.cuh", "kernels_common.cuh"),
-    "b16": ("batch.cuh", "kernels_common.cuh", "rnn_epilogue.cuh", "spmm_batch.cu"),
+    "b16": ("batch.cuh", "kernels_common.cuh", "rnn_epilogue.cuh", "spmm_batch.cu", "xres.cuh"),
+    "xres": ("xres.cuh", "kernels_common.cuh", "spmm_batch.cu", "batch.cuh", "rnn_epilogue.cuh"),
     "tc": ("tc.cuh", "tcgen05.cuh", "spmm_tc.cu"),
 }
 
 
 def call_sources(call: str):
-    """The csrc files the kernels of a bench call (e.g. fc6_spmm_b256) come from."""
+    """The csrc files the kernels of a bench call (e.g. fc6_spmm_b256, or
+    fc6_tc_b256 for the opt-in tensor-core path) come from."""
     if call.endswith("_encode"):
         kind = "encode"
+    elif "_tc_b" in call:
+        kind = "tc"
     else:
         b = int(call.rsplit("_b", 1)[1])
-        kind = "b1" if b == 1 else ("b16" if b < 33 else "tc")
+        kind = "b1" if b == 1 else ("b16" if b <= 16 else "xres")
     return tuple(sorted(_COMMON_SOURCES + _CALL_SOURCES[kind]))
 
 
@@ -350,13 +352,20 @@ def roofline(wl, di, dom, dom_ms, achieved, peak, peak_kind, tpeak, tpeak_kind, 
                         " not algorithmic work); that work, not HBM, binds it. gather_equiv_frac = the"
                         " (kept weight, column) operands per second against the CUDA-core gather bound"
                         " of 128 B/clk/SM"}
-    return {"bound": "hbm", "kernel": dom, "achieved": round(achieved, 1),
-            "peak": peak, "peak_kind": peak_kind, "unit": "GB/s", "frac": round(achieved / peak, 4),
-            "frac_of_nominal_8000": round(achieved / 8000.0, 4), "share_of_step": share,
-            "traffic": traffic,
-            "note": "achieved = algorithmic bytes per launch (values + offsets + row metadata + X + Y,"
-                    " or dense W + encoding for encode) / mean launch time; for batch > 4 the"
-                    " on-chip activation gather, not HBM, binds (parts[].gather_frac)"}
+    out = {"bound": "hbm", "kernel": dom, "achieved": round(achieved, 1),
+           "peak": peak, "peak_kind": peak_kind, "unit": "GB/s", "frac": round(achieved / peak, 4),
+           "frac_of_nominal_8000": round(achieved / 8000.0, 4), "share_of_step": share,
+           "traffic": traffic,
+           "note": "achieved = algorithmic bytes per launch (values + offsets + row metadata + X + Y,"
+                   " or dense W + encoding for encode) / median launch time; for batch > 4 the"
+                   " on-chip activation gather, not HBM, binds: gather_frac"}
+    if kind == "spmm" and b > 4:
+        nnzb = wl.mats[mi]["info"]["nnzb"]
+        out["gather_frac"] = round(nnzb * b * 4 / (dom_ms * 1e-3) / 1e9 / gather_peak, 4)
+        out["gather_peak_gbs"] = round(gather_peak, 1)
+        out["binding"] = ("on-chip activation gather: every (kept weight, batch column) product reads a 4-byte "
+                          "activation from shared memory, at most 128 B/clk/SM")
+    return out
 
 
 # ----------------------------------------------------------------------------- GPU arm
@@ -481,20 +490,35 @@ def run_gpu(args, world, rank, local):
     elapsed_ms = max_over_ranks(elapsed_ms, world)
     ms_per_step = elapsed_ms / args.steps
 
+    # the same step without programmatic dependent launch: every kernel starts
+    # only when the previous one has finished
+    darb.darb_set_pdl(False)
+    try:
+        graphs_off = [capture(torch, lambda s=s: [wl.launch(c, s, None) for c in wl.calls]) for s in range(NSETS)]
+        for s in range(args.warmup):
+            graphs_off[s % NSETS].replay()
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize()
+        a.record(stream)
+        for s in range(args.steps):
+            graphs_off[s % NSETS].replay()
+        b.record(stream)
+        torch.cuda.synchronize()
+        ms_pdl_off = a.elapsed_time(b) / args.steps
+    finally:
+        darb.darb_set_pdl(True)
+    wl.check_encode()
+
     # per-call breakdown: each call of the step launched back to back over the
-    # rotating buffer sets (still cold in L2), from a graph, events at both ends
+    # rotating buffer sets (still cold in L2), from a graph replayed REPEATS
+    # times with events around each replay: median (and mean) per call
     per_call = np.zeros(ncalls)
+    per_call_mean = np.zeros(ncalls)
     reps = max(1, args.steps // NSETS)
     for i, c in enumerate(wl.calls):
         g = capture(torch, lambda c=c: [wl.launch(c, s, None) for _ in range(reps) for s in range(NSETS)])
-        g.replay()
-        a = torch.cuda.Event(enable_timing=True)
-        b = torch.cuda.Event(enable_timing=True)
-        a.record(stream)
-        g.replay()
-        b.record(stream)
-        torch.cuda.synchronize()
-        per_call[i] = a.elapsed_time(b) / (reps * NSETS)
+        per_call[i], per_call_mean[i] = replay_times(torch, g, stream, reps * NSETS)
     wl.check_encode()
     peak, peak_kind = measured_peaks()
     clocks = nv.summary() or clk.summary()
@@ -511,7 +535,8 @@ def run_gpu(args, world, rank, local):
         gbs = nbytes / sec / 1e9
         path, kernels = wl.paths[i]
         part = {"call": name, "path": path, "kernels": kernels, "bytes": int(nbytes),
-                "us": round(per_call[i] * 1e3, 3), "gbs": round(gbs, 1), "hbm_frac": round(gbs / peak, 4)}
+                "us": round(per_call[i] * 1e3, 3), "us_mean": round(per_call_mean[i] * 1e3, 3),
+                "gbs": round(gbs, 1), "hbm_frac": round(gbs / peak, 4)}
         if kind == "spmm":
             nnzb = wl.mats[mi]["info"]["nnzb"]
             part["gflops"] = round(2 * nnzb * b / sec / 1e9, 1)
@@ -549,12 +574,19 @@ def run_gpu(args, world, rank, local):
                              step_ms_sum, gather_peak),
         "gather_peak_gbs": round(gather_peak, 1),
         "parts": parts,
-        "parts_note": "per call: K launches of that call alone, back to back on rotating cold buffers,"
-                      " replayed from a CUDA graph",
+        "parts_note": f"per call: {reps * NSETS} launches of that call alone, back to back on rotating cold"
+                      f" buffers, from a CUDA graph replayed {REPEATS} times: us = median over the replays,"
+                      " us_mean = their mean",
+        "pdl_off": {"ms_per_step": round(ms_pdl_off, 5),
+                    "value": round(world * wl.step_bytes / (ms_pdl_off * 1e-3) / 1e9, 2), "unit": "GB/s",
+                    "note": "the same step captured with programmatic dependent launch off (darb_set_pdl)"},
         "timing": "CUDA-graph replay of whole steps (one graph per buffer set); CUDA events on the stream",
         "gpu_launches": wl.step_launches * args.steps,
         "clocks": clocks,
     }
+    if not only:
+        result["tensor_cores"] = run_tensor(torch, darb, wl, stream)
+        result["gemv_1024"] = run_gemv_1024(torch, darb, synth, peak, stream)
     if not args.no_rnn and not only:
         result["rnn"] = run_rnn(torch, darb, synth, peak)
         result["assign"] = run_assign(torch, darb, wl, peak)
@@ -564,6 +596,96 @@ def run_gpu(args, world, rank, local):
         result["e2e"] = run_e2e(args, wl, torch, darb)
     wl.close()
     return result
+
+
+REPEATS = 10   # replays of a per-call graph, for the median
+
+
+def replay_times(torch, g, stream, calls, repeats=REPEATS):
+    """Median and mean time per call (ms) of a graph holding `calls` launches,
+    replayed `repeats` times after one warm-up replay, CUDA events around each."""
+    g.replay()
+    times = []
+    for _ in range(repeats):
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        g.replay()
+        b.record(stream)
+        torch.cuda.synchronize()
+        times.append(a.elapsed_time(b) / calls)
+    return statistics.median(times), statistics.mean(times)
+
+
+def run_tensor(torch, darb, wl, stream):
+    """The opt-in tensor-core path (darb_spmm_ex with DARB_PATH_TENSOR_CORES;
+    not darb_spmm, not the paper's per-block selection: densified tiles, X split
+    into two bf16 parts) on the step's wide products, timed like `parts`."""
+    out = {}
+    tpeak, tpeak_kind = measured_bf16_tflops()
+    for mi, mat in enumerate(wl.mats):
+        for b in (64, 256):
+            def launch(b=b, mi=mi):
+                for s in range(NSETS):
+                    st = wl.sets[s]
+                    darb.darb_spmm_ex(st["spmm"][(mi, b)], st["X"][(mi, b)], st["Y"][(mi, b)],
+                                      darb.PATH_TENSOR_CORES)
+            launch()
+            torch.cuda.synchronize()
+            g = capture(torch, launch)
+            med, mean = replay_times(torch, g, stream, NSETS)
+            nbytes = spmm_bytes(mat["info"], b)
+            tfl = tensor_flops(mat, b) / (med * 1e-3) / 1e12
+            out[f"{'fc6' if mi == 0 else 'fc7'}_tc_b{b}"] = {
+                "us": round(med * 1e3, 3), "us_mean": round(mean * 1e3, 3),
+                "gbs_algorithmic": round(nbytes / (med * 1e-3) / 1e9, 1),
+                "executed_tensor_tflops": round(tfl, 1), "executed_tensor_frac": round(tfl / tpeak, 4),
+                "tensor_peak_kind": tpeak_kind}
+    wl.check_encode()
+    out["note"] = ("opt-in densified-tile product on the tensor cores (darb_spmm_ex, DARB_PATH_TENSOR_CORES): "
+                   "executed FLOPs = 2 x 2 x rows x cols x batch (zeros and both bf16 parts of X), not "
+                   "algorithmic work; darb_spmm itself never takes this path")
+    return out
+
+
+def run_gemv_1024(torch, darb, synth, peak, stream, nsets=48):
+    """Workload gemv_1024 (a 1024 x 1024 fp32 matrix, per-row block sizes from
+    {8, 16, 32, 64}): DARB encode, then the product at batch 1.  The dense
+    matrices (4 MiB each) rotate over `nsets` sets (> L2), so every call reads
+    cold HBM; per call: median over replays, as `parts`."""
+    wl1 = synth.WORKLOADS["gemv_1024"]
+    rows, cols = wl1.shapes[0]
+    dev = torch.device("cuda", torch.cuda.current_device())
+    _, stored, m = synth.matrix(wl1, 0)
+    W0 = torch.from_numpy(stored).to(dev)
+    h0 = darb.darb_encode(W0, m)
+    info = darb.darb_info(h0)
+    val, off, _, mm = darb.darb_export(h0)
+    Ws = [W0.clone() for _ in range(nsets)]
+    hs = [darb.darb_import(val, off, mm, darb.F32, rows, cols) for _ in range(nsets)]
+    Xs = [torch.from_numpy(synth.activations(cols, 1, seed=wl1.seed, sub=s)).to(dev) for s in range(nsets)]
+    Ys = [torch.empty((rows, 1), device=dev) for _ in range(nsets)]
+    enc_b, spmm_b = encode_bytes(info), spmm_bytes(info, 1)
+    out = {"rows": rows, "cols": cols, "dtype": "f32", "nnzb": info["nnzb"],
+           "pruning_ratio": round(rows * cols / info["nnzb"], 2)}
+    calls = {"encode": lambda s: darb.darb_reencode(hs[s], Ws[s]),
+             "spmm_b1": lambda s: darb.darb_spmm(hs[s], Xs[s], Ys[s]),
+             "step": lambda s: (darb.darb_reencode(hs[s], Ws[s]), darb.darb_spmm(hs[s], Xs[s], Ys[s]))}
+    for name, fn in calls.items():
+        for s in range(nsets):
+            fn(s)
+        torch.cuda.synchronize()
+        g = capture(torch, lambda fn=fn: [fn(s) for s in range(nsets)])
+        med, mean = replay_times(torch, g, stream, nsets)
+        nbytes = {"encode": enc_b, "spmm_b1": spmm_b, "step": enc_b + spmm_b}[name]
+        gbs = nbytes / (med * 1e-3) / 1e9
+        out[name] = {"us": round(med * 1e3, 3), "us_mean": round(mean * 1e3, 3), "bytes": int(nbytes),
+                     "gbs": round(gbs, 1), "hbm_frac": round(gbs / peak, 4)}
+    for h in hs:
+        darb.darb_sync_status(h)
+        darb.darb_destroy(h)
+    darb.darb_destroy(h0)
+    return out
 
 
 def run_assign(torch, darb, wl, peak, reps=3):
@@ -651,13 +773,14 @@ def run_baselines(torch, darb, wl, reps=20):
                 t_cols = timed(lambda: call(XT, YT, baselines.DENSE_COLS))
                 row[f"{fmt}_us"] = round(min(t_rows, t_cols), 2)
                 row[f"{fmt}_layout"] = "rows" if t_rows <= t_cols else "cols"
-            row["darb_speedup_vs"] = {f: round(row[f"{f}_us"] / t_darb, 2) for f in ("csr", "bsr4", "bsr8")}
             entry[f"b{B}"] = row
         out[name] = entry
-    out["note"] = ("cuSPARSE SpMM, fp32 values and compute, in the faster of the two dense layouts (batch "
-                   "contiguous, or each batch column contiguous; the transposition is not timed); CSR = DARB's "
-                   "kept weights; BSR = the largest-L1 bs x bs blocks of the same W at the same kept-weight "
-                   "count; darb_spmm with bf16 values as in the step; every matrix L2-resident")
+    out["note"] = ("vendor-library figures, not a tuned block-sparse or CSR kernel and not the paper's "
+                   "Sec. 4.2 comparison: cuSPARSE SpMM with fp32 values (DARB: bf16 values, so the bytes "
+                   "differ), in the faster of the two dense layouts (batch contiguous, or each batch column "
+                   "contiguous; the transposition is not timed); CSR = DARB's kept weights; BSR = the "
+                   "largest-L1 bs x bs blocks of the same W at the same kept-weight count; every matrix "
+                   "L2-resident")
     return out
 
 
@@ -857,60 +980,113 @@ def run_e2e(args, wl, torch, darb):
 
 
 # ----------------------------------------------------------------------------- CPU oracle arm
-def oracle_sample(budget_s: float = 12.0):
-    """The oracle as it stands on a bounded sample of the same workload: encode of
-    FC7 and its product at batch 1 and 16.  Returns (GB/s, seconds, cores, sample)."""
-    import oracle
-    from paper_1911_08020_gb300 import synth
-    wl = synth.WORKLOADS[WORKLOAD]
-    _, bits, m = synth.matrix(wl, 1)
-    rows, cols = wl.shapes[1]
-    cores = oracle.set_threads(0)
-    X1 = synth.activations(cols, 1, seed=wl.seed, sub=91)
-    X16 = synth.activations(cols, 16, seed=wl.seed, sub=92)
-    total_bytes, total_s, reps = 0, 0.0, 0
-    while total_s < budget_s or reps == 0:
+def cpu_model() -> str:
+    """The host CPU's name, from /proc/cpuinfo (x86 'model name', or the Arm
+    implementer / part numbers) or lscpu."""
+    try:
+        with open("/proc/cpuinfo") as f:
+            info = f.read()
+        for key in ("model name", "Model name"):
+            for ln in info.splitlines():
+                if ln.startswith(key):
+                    return ln.split(":", 1)[1].strip()
+        impl = [ln.split(":", 1)[1].strip() for ln in info.splitlines() if ln.startswith("CPU implementer")]
+        part = [ln.split(":", 1)[1].strip() for ln in info.splitlines() if ln.startswith("CPU part")]
+        if impl and part:
+            return f"Arm implementer {impl[0]} part {part[0]}"
+    except OSError:
+        pass
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for ln in out.splitlines():
+            if ln.startswith("Model name"):
+                return ln.split(":", 1)[1].strip()
+    except (OSError, subprocess.SubprocessError):
+        pass
+    return "unknown"
+
+
+class OracleStep:
+    """The step the GPU arm times -- BMWM encode of FC6 and FC7, then the
+    product of each at batch 1, 16, 64 and 256 -- run by the CPU oracle as it
+    stands: its encoder, and its fp32-accumulate product loop (OpenMP over
+    rows).  Bytes: the same algorithmic bytes as the GPU step."""
+
+    def __init__(self):
+        import oracle
+        from paper_1911_08020_gb300 import synth
+        self.oracle = oracle
+        wl = synth.WORKLOADS[WORKLOAD]
+        self.mats = []
+        self.bytes = 0
+        for i, (rows, cols) in enumerate(wl.shapes):
+            _, bits, m = synth.matrix(wl, i)
+            X = {b: synth.activations(cols, b, seed=wl.seed, sub=90 + b) for b in BATCHES}
+            nnzb = int(oracle.block_pointers(m, cols)[-1])
+            info = {"rows": rows, "cols": cols, "wtype": 1, "value_bytes": nnzb * 2,
+                    "offset_bytes": sum(-(-cols // int(x)) * (4 if x <= 16 else 8) for x in m) // 8,
+                    "meta_bytes": rows * 6}
+            self.bytes += encode_bytes(info) + sum(spmm_bytes(info, b) for b in BATCHES)
+            self.mats.append((bits, m, X))
+
+    def run(self) -> float:
+        """One step; returns its wall time in seconds."""
         t0 = time.perf_counter()
-        enc = oracle.encode(bits, m, "bf16")
-        oracle.darb_spmm(enc, X1)
-        oracle.darb_spmm(enc, X16)
-        total_s += time.perf_counter() - t0
-        nnzb = int(enc.blk_ptr[-1])
-        vb = nnzb * 2
-        ob = sum(-(-cols // int(x)) * (4 if x <= 16 else 8) for x in m) // 8
-        meta = rows * 6
-        total_bytes += (rows * cols * 2 + vb + ob + meta) + sum(
-            vb + ob + meta + cols * b * 4 + rows * b * 4 for b in (1, 16))
-        reps += 1
-        if reps >= 2000:
-            break
-    sample = f"FC7 4096x4096 bf16: oracle encode + darb_spmm at batch 1 and 16, x{reps}"
-    return total_bytes / total_s / 1e9, total_s, cores, sample
+        encs = [self.oracle.encode(bits, m, "bf16") for bits, m, _ in self.mats]
+        for b in BATCHES:
+            for enc, (_, _, X) in zip(encs, self.mats):
+                self.oracle.darb_spmm_f32(enc, X[b])
+        return time.perf_counter() - t0
+
+
+def cpu_protocol(runs: int = 5):
+    """The oracle on the GPU step's calls at 1 thread and at nproc threads,
+    median of `runs` steps each, with the CPU named."""
+    import oracle
+    oracle.build()
+    step = OracleStep()
+    nproc = os.cpu_count() or 1
+    out = {"cpu_model": cpu_model(), "nproc": nproc, "runs": runs, "bytes_per_step": int(step.bytes)}
+    for threads in (1, nproc):
+        used = oracle.set_threads(threads)
+        step.run()   # warm-up: page in, first-touch
+        times = [step.run() for _ in range(runs)]
+        med = statistics.median(times)
+        out[f"threads_{threads}" if threads == 1 else "threads_nproc"] = {
+            "threads": used, "median_s": round(med, 4), "min_s": round(min(times), 4),
+            "gbs": round(step.bytes / med / 1e9, 3)}
+    oracle.set_threads(nproc)
+    out["sample"] = ("the whole FC6 + FC7 step: oracle encode (bf16) + oracle darb_spmm_f32 (fp32 accumulate) "
+                     "at batch 1/16/64/256, median of %d steps" % runs)
+    return out
 
 
 def run_reference(args, world, rank):
+    """The reference arm: the CPU oracle as it stands (the paper ships no code)
+    runs the GPU arm's step at nproc threads; `value` = the step's algorithmic
+    bytes over the mean step time."""
     if rank != 0:
         return None
     import oracle
     oracle.build()
-    per_step = []
-    for s in range(args.warmup + args.steps):
-        gbs, secs, cores, sample = oracle_sample(
-            budget_s=max(0.2, args.cpu_seconds / max(1, args.steps + args.warmup)))
-        if s >= args.warmup:
-            per_step.append(secs)
-        last = (gbs, cores, sample)
-    gbs, cores, sample = last
-    ms = 1e3 * statistics.mean(per_step)
+    step = OracleStep()
+    cores = oracle.set_threads(os.cpu_count() or 1)
+    for _ in range(args.warmup):
+        step.run()
+    times = [step.run() for _ in range(args.steps)]
+    ms = 1e3 * statistics.mean(times)
+    gbs = step.bytes / (ms * 1e-3) / 1e9
+    sample = ("the whole FC6 + FC7 step per timed step: oracle encode (bf16) + oracle darb_spmm_f32 (fp32 "
+              "accumulate) at batch 1/16/64/256")
     return {
         "metric": METRIC, "value": round(gbs, 3), "unit": "GB/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms, 3),
-        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
         "data": "synthetic", "impl": "reference",
         "config": {"workload": "fc6_fc7_4096x9216_4096x4096_bf16_weights",
-                   "sample": sample, "parallelism": "cpu"},
+                   "batches": list(BATCHES), "sample": sample, "parallelism": "cpu"},
         "cpu_baseline": {"value": round(gbs, 3), "unit": "GB/s", "cores": cores, "kind": "oracle",
-                         "sample": sample},
+                         "sample": sample, "cpu_model": cpu_model()},
         "e2e": {"value": round(gbs, 3), "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
 
@@ -926,11 +1102,12 @@ def main():
     res = run_gpu(args, world, rank, local)
     if rank == 0:
         if not args.no_cpu and world == 1:
-            import oracle
-            oracle.build()
-            gbs, secs, cores, sample = oracle_sample()
-            res["cpu_baseline"] = {"value": round(gbs, 3), "unit": "GB/s", "cores": cores,
-                                   "kind": "oracle", "sample": sample, "seconds": round(secs, 2)}
+            cp = cpu_protocol()
+            res["cpu_baseline"] = {"value": cp["threads_nproc"]["gbs"], "unit": "GB/s",
+                                   "cores": cp["threads_nproc"]["threads"], "kind": "oracle",
+                                   "sample": cp["sample"], "cpu_model": cp["cpu_model"],
+                                   "threads_1": cp["threads_1"], "threads_nproc": cp["threads_nproc"],
+                                   "same_step_as_gpu": True}
         print(json.dumps(res), flush=True)
     if world > 1:
         import torch.distributed as dist

@@ -350,6 +350,15 @@ DARB_API darb_status_t darb_import(const void *val, const uint8_t *off, const in
                           darb_dtype_t wtype, int64_t rows, int64_t cols, darb_handle_t *out,
                           cudaStream_t stream);
 
+/* Whether the library's kernels are launched with programmatic dependent
+ * launch (PDL: a kernel may start its prologue, and read the handle's
+ * immutable data, while the previous kernel on the stream drains; its reads
+ * of X and writes of Y still wait for that kernel).  Process wide, on by
+ * default; applies to launches made after the call (a CUDA graph keeps what
+ * it captured).  For measuring the overlap; results are the same either way.
+ * The paper has no counterpart.  Always DARB_OK.                             */
+DARB_API darb_status_t darb_set_pdl(int enabled);
+
 /* Release a handle and all device memory it owns; NULL is a no-op.  Waits for
  * the device to finish using it.                                              */
 DARB_API darb_status_t darb_destroy(darb_handle_t h);

@@ -12,6 +12,7 @@ Functions (each follows the passage cited in ``darb_oracle.c``):
 * ``encode(W, m, dtype)``                              BMWM, Sec. 3.1 / 3.2
 * ``masked_dense(enc, cols)``                          the dense M (.) W
 * ``darb_spmm(enc, X)``                                y = W_darb X in fp64
+* ``darb_spmm_f32(enc, X)``                            the same sum in fp32, for timing only
 * ``lstm_step(enc, I, H, x, h, c, bias)`` / ``gru_step(enc, I, H, x, h, b_ih, b_hh)``
 """
 from __future__ import annotations
@@ -73,11 +74,12 @@ def load_library(path: str):
     lib.oracle_encode_bf16.argtypes = [P, I64, I64, I64, P, P, P, P]
     lib.oracle_masked_dense.argtypes = [P, P, P, P, I64, I64, P]
     lib.oracle_darb_spmm.argtypes = [P, P, P, P, I64, I64, P, I64, I64, P, I64, P]
+    lib.oracle_darb_spmm_f32_timed.argtypes = [P, P, P, P, I64, I64, P, I64, I64, P, I64]
     lib.oracle_lstm_step.argtypes = [P, P, P, P, I64, I64, I64, P, P, P, P, P, P, P]
     lib.oracle_gru_step.argtypes = [P, P, P, P, I64, I64, I64, P, P, P, P, P, P]
     for f in ("oracle_assign_block_sizes", "oracle_topk_row_nnz_f32", "oracle_topk_row_nnz_bf16",
               "oracle_block_pointers", "oracle_encode_f32",
-              "oracle_encode_bf16", "oracle_masked_dense", "oracle_darb_spmm",
+              "oracle_encode_bf16", "oracle_masked_dense", "oracle_darb_spmm", "oracle_darb_spmm_f32_timed",
               "oracle_lstm_step", "oracle_gru_step"):
         getattr(lib, f).restype = ctypes.c_int
     return lib
@@ -188,6 +190,21 @@ def darb_spmm(enc: Encoding, X: np.ndarray, with_absdot: bool = False):
                                     enc.cols, _p(X), batch, batch, _p(Y), batch,
                                     _p(A) if A is not None else None), "darb_spmm")
     return (Y, A) if with_absdot else Y
+
+
+def darb_spmm_f32(enc: Encoding, X: np.ndarray, values_f32: np.ndarray | None = None):
+    """The same product in fp32 (fp32 accumulate, block order): the loop timed
+    as the CPU baseline.  Never a reference value: parity is against darb_spmm.
+    values_f32 may pass the kept values already widened to float32."""
+    X = np.ascontiguousarray(X, dtype=np.float32)
+    if X.ndim == 1:
+        X = X[:, None]
+    batch = X.shape[1]
+    Y = np.empty((enc.rows, batch), dtype=np.float32)
+    v = values_f32 if values_f32 is not None else enc.values_f64().astype(np.float32)
+    _check(_load().oracle_darb_spmm_f32_timed(_p(v), _p(enc.off), _p(enc.blk_ptr), _p(enc.m), enc.rows,
+                                              enc.cols, _p(X), batch, batch, _p(Y), batch), "darb_spmm_f32")
+    return Y
 
 
 def lstm_step(enc: Encoding, I: int, H: int, x, h_prev, c_prev, bias=None):

@@ -251,6 +251,30 @@ int oracle_darb_spmm(const double *val, const uint8_t *off, const int64_t *blk_p
     return bad ? OR_INVALID : OR_OK;
 }
 
+/* The same sum (Sec. 3.2, Fig. 6(b)) in single precision, for timing the
+ * oracle as a CPU baseline only (never used as a reference value): kept values
+ * widened to float, X float, one float accumulator per output, added in block
+ * order; OpenMP over rows.                                                   */
+int oracle_darb_spmm_f32_timed(const float *val, const uint8_t *off, const int64_t *blk_ptr,
+                               const int32_t *m, int64_t rows, int64_t cols, const float *X,
+                               int64_t ldx, int64_t batch, float *Y, int64_t ldy) {
+    if (!val || !off || !blk_ptr || !m || !X || !Y || rows <= 0 || cols <= 0 || batch <= 0 ||
+        ldx < batch || ldy < batch)
+        return OR_INVALID;
+    int bad = 0;
+    _Pragma("omp parallel for schedule(static) reduction(|:bad)")
+    for (int64_t r = 0; r < rows; ++r) {
+        for (int64_t b = 0; b < batch; ++b) Y[r * ldy + b] = 0.0f;
+        for (int64_t p = blk_ptr[r]; p < blk_ptr[r + 1]; ++p) {
+            int64_t j = p - blk_ptr[r];
+            int64_t k = j * m[r] + off[p];
+            if (off[p] >= m[r] || k >= cols) { bad = 1; break; }
+            for (int64_t b = 0; b < batch; ++b) Y[r * ldy + b] += val[p] * X[k * ldx + b];
+        }
+    }
+    return bad ? OR_INVALID : OR_OK;
+}
+
 static double sigmoid(double v) { return 1.0 / (1.0 + exp(-v)); }
 
 /* One LSTM step.  The gate matrix is 4H x (I+H), its input the stacked column

@@ -85,7 +85,7 @@ def build(force: bool = False, ptxas_verbose: bool = False) -> str:
     srcs = SOURCES + BASE_SOURCES
     with cf.ThreadPoolExecutor(max_workers=len(srcs)) as ex:
         objs = dict(zip(srcs, ex.map(lambda s: _compile(s, ptxas_verbose), srcs)))
-    _link([objs[s] for s in SOURCES], LIB)
+    _link([objs[s] for s in SOURCES], LIB, ["-ldl"])   # NVTX loads a profiler's injection library
     libdir = _cuda_lib_dir()
     _link([objs[s] for s in BASE_SOURCES], BASE_LIB, ["-L" + libdir, "-lcusparse", "-Xlinker", "-rpath=" + libdir])
     return LIB

@@ -2,7 +2,9 @@
 // handle lifetime, the binned device layout, and kernel launches.
 #include "darb.h"
 #include "darb_internal.h"
+#include "launch.cuh"
 #include "tma.cuh"
+#include "trace.h"
 
 #include <algorithm>
 #include <cstdlib>
@@ -491,6 +493,7 @@ const char *darb_status_string(darb_status_t s) {
 
 darb_status_t darb_assign_block_sizes(const int64_t *row_nnz, int64_t rows, int64_t cols,
                                       int32_t m_min, int32_t m_max, int32_t *m_out) {
+    DARB_TRACE("darb_assign_block_sizes");
     if (row_nnz == nullptr || m_out == nullptr || rows <= 0 || cols <= 0 || m_min < 1 ||
         m_max < m_min || m_max > DARB_MAX_BLOCK)
         return DARB_ERR_INVALID_ARG;
@@ -523,6 +526,7 @@ darb_status_t darb_assign_block_sizes(const int64_t *row_nnz, int64_t rows, int6
 
 darb_status_t darb_encode(const void *W, darb_dtype_t wtype, int64_t rows, int64_t cols,
                           int64_t ldw, const int32_t *m, darb_handle_t *out, cudaStream_t stream) {
+    DARB_TRACE("darb_encode");
     if (out == nullptr) return DARB_ERR_INVALID_ARG;
     *out = nullptr;
     if (W == nullptr || !valid_dtype(wtype) || ldw < cols) return DARB_ERR_INVALID_ARG;
@@ -560,6 +564,7 @@ darb_status_t darb_encode(const void *W, darb_dtype_t wtype, int64_t rows, int64
 }
 
 darb_status_t darb_reencode(darb_handle_t h, const void *W, int64_t ldw, cudaStream_t stream) {
+    DARB_TRACE("darb_reencode");
     if (!live(h) || W == nullptr || ldw < h->cols) return DARB_ERR_INVALID_ARG;
     const size_t esz = h->wtype == DARB_BF16 ? 2 : 4;
     if (reinterpret_cast<uintptr_t>(W) % esz != 0) return DARB_ERR_INVALID_ARG;
@@ -580,6 +585,7 @@ darb_status_t darb_reencode(darb_handle_t h, const void *W, int64_t ldw, cudaStr
 }
 
 darb_status_t darb_sync_status(darb_handle_t h, cudaStream_t stream) {
+    DARB_TRACE("darb_sync_status");
     if (!live(h)) return DARB_ERR_INVALID_ARG;
     int32_t bits = 0;
     cudaError_t e = cudaMemcpyAsync(&bits, h->d_status, 4, cudaMemcpyDeviceToHost, stream);
@@ -592,11 +598,13 @@ darb_status_t darb_sync_status(darb_handle_t h, cudaStream_t stream) {
 
 darb_status_t darb_spmm(darb_handle_t h, const float *X, int64_t ldx, int64_t batch, float *Y,
                         int64_t ldy, cudaStream_t stream) {
+    DARB_TRACE("darb_spmm");
     return darb_spmm_ex(h, X, ldx, batch, Y, ldy, DARB_PATH_AUTO, stream);
 }
 
 darb_status_t darb_spmm_ex(darb_handle_t h, const float *X, int64_t ldx, int64_t batch, float *Y,
                            int64_t ldy, darb_path_t path, cudaStream_t stream) {
+    DARB_TRACE("darb_spmm_ex");
     if (path != DARB_PATH_AUTO && path != DARB_PATH_CUDA_CORES && path != DARB_PATH_TENSOR_CORES)
         return DARB_ERR_INVALID_ARG;
     if (!live(h) || X == nullptr || Y == nullptr || batch <= 0 || ldx < batch || ldy < batch)
@@ -622,6 +630,7 @@ darb_status_t darb_spmm_ex(darb_handle_t h, const float *X, int64_t ldx, int64_t
 darb_status_t darb_assign_from_weights(const void *W, darb_dtype_t wtype, int64_t rows, int64_t cols, int64_t ldw,
                                        int64_t keep, int32_t m_min, int32_t m_max, int64_t *row_nnz_out,
                                        int32_t *m_out, cudaStream_t stream) {
+    DARB_TRACE("darb_assign_from_weights");
     if (W == nullptr || m_out == nullptr || !valid_dtype(wtype)) return DARB_ERR_INVALID_ARG;
     if (rows <= 0 || cols <= 0 || rows > kMaxDim || cols > kMaxDim || ldw < cols) return DARB_ERR_INVALID_ARG;
     if (m_min < 1 || m_max < m_min || m_max > DARB_MAX_BLOCK) return DARB_ERR_INVALID_ARG;
@@ -677,6 +686,7 @@ darb_status_t darb_assign_from_weights(const void *W, darb_dtype_t wtype, int64_
 }
 
 darb_status_t darb_spmm_path(darb_handle_t h, int64_t batch, darb_path_t *path, int32_t *kernels) {
+    DARB_TRACE("darb_spmm_path");
     if (!live(h) || batch <= 0 || path == nullptr || kernels == nullptr) return DARB_ERR_INVALID_ARG;
     // darb_spmm always takes the CUDA-core gather: one kernel per call
     *path = DARB_PATH_CUDA_CORES;
@@ -685,6 +695,7 @@ darb_status_t darb_spmm_path(darb_handle_t h, int64_t batch, darb_path_t *path, 
 }
 
 darb_status_t darb_rnn_reserve(darb_handle_t h, int64_t max_batch) {
+    DARB_TRACE("darb_rnn_reserve");
     if (!live(h) || max_batch <= 0 || max_batch > kMaxBatch) return DARB_ERR_INVALID_ARG;
     // GRU needs the larger gate buffer; the smallest tile gives the most counters
     const int64_t units = h->rows;   // upper bound on H for either cell
@@ -708,6 +719,7 @@ static darb_status_t check_step(darb_handle_t h, int64_t I, int64_t H, int64_t B
 darb_status_t darb_lstm_step(darb_handle_t h, int64_t I, int64_t H, int64_t B, const float *x,
                              const float *h_prev, const float *c_prev, const float *bias,
                              float *h_out, float *c_out, cudaStream_t stream) {
+    DARB_TRACE("darb_lstm_step");
     darb_status_t st = check_step(h, I, H, B, 4, x, h_prev);
     if (st != DARB_OK) return st;
     if (c_prev == nullptr || h_out == nullptr || c_out == nullptr) return DARB_ERR_INVALID_ARG;
@@ -728,6 +740,7 @@ darb_status_t darb_lstm_step(darb_handle_t h, int64_t I, int64_t H, int64_t B, c
 darb_status_t darb_gru_step(darb_handle_t h, int64_t I, int64_t H, int64_t B, const float *x,
                             const float *h_prev, const float *b_ih, const float *b_hh,
                             float *h_out, cudaStream_t stream) {
+    DARB_TRACE("darb_gru_step");
     darb_status_t st = check_step(h, I, H, B, 3, x, h_prev);
     if (st != DARB_OK) return st;
     if (h_out == nullptr) return DARB_ERR_INVALID_ARG;
@@ -756,6 +769,7 @@ static darb_status_t sequence_status(cudaError_t e) {
 darb_status_t darb_lstm_sequence(darb_handle_t h, int64_t T, int64_t I, int64_t H, int64_t B, const float *x_seq,
                                  const float *h0, const float *c0, const float *bias, float *h_seq, float *c_seq,
                                  float *c_last, cudaStream_t stream) {
+    DARB_TRACE("darb_lstm_sequence");
     // x_seq may be NULL when there are no steps
     darb_status_t st = check_step(h, I, H, B, 4, T > 0 ? x_seq : h0, h0);
     if (st != DARB_OK) return st;
@@ -782,6 +796,7 @@ darb_status_t darb_lstm_sequence(darb_handle_t h, int64_t T, int64_t I, int64_t 
 darb_status_t darb_gru_sequence(darb_handle_t h, int64_t T, int64_t I, int64_t H, int64_t B, const float *x_seq,
                                 const float *h0, const float *b_ih, const float *b_hh, float *h_seq,
                                 cudaStream_t stream) {
+    DARB_TRACE("darb_gru_sequence");
     darb_status_t st = check_step(h, I, H, B, 3, T > 0 ? x_seq : h0, h0);
     if (st != DARB_OK) return st;
     if (T < 0 || (T > 0 && h_seq == nullptr)) return DARB_ERR_INVALID_ARG;
@@ -798,6 +813,7 @@ darb_status_t darb_gru_sequence(darb_handle_t h, int64_t T, int64_t I, int64_t H
 }
 
 darb_status_t darb_info(darb_handle_t h, darb_info_t *info) {
+    DARB_TRACE("darb_info");
     if (!live(h) || info == nullptr) return DARB_ERR_INVALID_ARG;
     darb_info_t r{};
     r.rows = h->rows;
@@ -825,6 +841,7 @@ darb_status_t darb_info(darb_handle_t h, darb_info_t *info) {
 }
 
 darb_status_t darb_export(darb_handle_t h, void *val, uint8_t *off, int64_t *blk_ptr, int32_t *m) {
+    DARB_TRACE("darb_export");
     if (!live(h)) return DARB_ERR_INVALID_ARG;
     const size_t esz = h->wtype == DARB_BF16 ? 2 : 4;
     std::vector<uint8_t> hv;
@@ -870,6 +887,7 @@ darb_status_t darb_export(darb_handle_t h, void *val, uint8_t *off, int64_t *blk
 darb_status_t darb_import(const void *val, const uint8_t *off, const int32_t *m,
                           darb_dtype_t wtype, int64_t rows, int64_t cols, darb_handle_t *out,
                           cudaStream_t stream) {
+    DARB_TRACE("darb_import");
     if (out == nullptr) return DARB_ERR_INVALID_ARG;
     *out = nullptr;
     if (val == nullptr || off == nullptr || !valid_dtype(wtype)) return DARB_ERR_INVALID_ARG;
@@ -929,7 +947,14 @@ darb_status_t darb_import(const void *val, const uint8_t *off, const int32_t *m,
     return DARB_OK;
 }
 
+darb_status_t darb_set_pdl(int enabled) {
+    DARB_TRACE("darb_set_pdl");
+    darb::pdl_setting().store(enabled ? 1 : 0, std::memory_order_relaxed);
+    return DARB_OK;
+}
+
 darb_status_t darb_destroy(darb_handle_t h) {
+    DARB_TRACE("darb_destroy");
     if (h == nullptr) return DARB_OK;
     {
         std::lock_guard<std::mutex> lk(g_mu);

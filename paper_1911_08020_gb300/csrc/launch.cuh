@@ -7,12 +7,21 @@
 #include <cudaTypedefs.h>
 #include <cuda_runtime.h>
 
+#include <atomic>
 #include <map>
 #include <mutex>
 #include <tuple>
 #include <utility>
 
 namespace darb {
+
+// Whether kernels are launched with programmatic dependent launch (process
+// wide; darb_set_pdl).  On by default.
+inline std::atomic<int> &pdl_setting() {
+    static std::atomic<int> on{1};
+    return on;
+}
+inline bool pdl_enabled() { return pdl_setting().load(std::memory_order_relaxed) != 0; }
 
 // The calling thread's current device (0 if it cannot be read).
 inline int current_device() {
@@ -71,7 +80,7 @@ cudaError_t launch_ex(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t sm
         attr[n].val.clusterDim.z = 1;
         ++n;
     }
-    if (pdl) {
+    if (pdl && pdl_enabled()) {
         attr[n].id = cudaLaunchAttributeProgrammaticStreamSerialization;
         attr[n].val.programmaticStreamSerializationAllowed = 1;
         ++n;

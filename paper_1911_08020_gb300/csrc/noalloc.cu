@@ -12,6 +12,7 @@
 // time (or ever, apart from the array itself, which every GPU that loads the
 // library holds until the process exits).
 #include "darb.h"
+#include "trace.h"
 #include "darb_internal.h"
 
 #include <mutex>
@@ -56,6 +57,7 @@ extern "C" darb_status_t darb_lstm_step_noalloc(darb_handle_t h, int64_t I, int6
                                                 const float *x, const float *h_prev,
                                                 const float *c_prev, const float *bias,
                                                 float *h_out, float *c_out, cudaStream_t stream) {
+    DARB_TRACE("darb_lstm_step_noalloc");
     darb::Format f;
     darb_status_t st = darb::lstm_step_view(h, I, H, B, x, h_prev, c_prev, bias, h_out, c_out, &f);
     if (st != DARB_OK) return st;

@@ -704,7 +704,7 @@ cudaError_t launch_kw(const Format &f, const float *X, int64_t ldx, int64_t batc
         attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
         attr[1].val.programmaticStreamSerializationAllowed = 1;
         cfg.attrs = attr;
-        cfg.numAttrs = 2;
+        cfg.numAttrs = pdl_enabled() ? 2 : 1;
         e = cudaLaunchKernelEx(&cfg, tc_kernel<KW>, hmap, lmap, f, coop_split, p.nstages, p.N, batch, Y, ldy, pt,
                                arrive, early ? 1 : 0);
         if (e != cudaSuccess) {   // not launchable cooperatively here: the cluster split instead

@@ -69,6 +69,7 @@ def lib():
                 "darb_export": [P, P, P, P, P],
                 "darb_import": [P, P, P, ctypes.c_int, I64, I64, P, S],
                 "darb_destroy": [P],
+                "darb_set_pdl": [ctypes.c_int],
             }
             for name, args in sig.items():
                 fn = getattr(L, name)
@@ -306,3 +307,8 @@ def darb_destroy(h: Handle | None):
         return
     _check(lib().darb_destroy(h.ptr), "darb_destroy")
     h.ptr = None
+
+
+def darb_set_pdl(enabled: bool):
+    """Launch the library's kernels with (default) or without programmatic dependent launch."""
+    _check(lib().darb_set_pdl(1 if enabled else 0), "darb_set_pdl")

@@ -320,6 +320,28 @@ def check_product_random(orc, seed=5):
         np.testing.assert_allclose(A, np.abs(Wd) @ np.abs(X.astype(np.float64)), rtol=1e-14, atol=0)
 
 
+def check_product_f32_timed(orc, seed=11):
+    """The single-precision loop timed as the CPU baseline: exact on small
+    integer inputs (every partial sum is an exactly representable integer),
+    and within fp32 summation error of numpy's masked dense product in
+    float64 on Gaussian inputs (|err| <= n * 2^-24 * sum |w x|)."""
+    g = np.random.default_rng(seed)
+    for _ in range(10):
+        rows, cols, B = int(g.integers(1, 60)), int(g.integers(1, 300)), int(g.integers(1, 7))
+        m = g.integers(1, 65, size=rows).astype(np.int32)
+        Wi = g.integers(-8, 9, size=(rows, cols)).astype(np.float32)
+        Xi = g.integers(-5, 6, size=(cols, B)).astype(np.float32)
+        enc = orc.encode(Wi, m)
+        np.testing.assert_array_equal(orc.darb_spmm_f32(enc, Xi), _numpy_masked(enc) @ Xi.astype(np.float64))
+        W = g.standard_normal((rows, cols)).astype(np.float32)
+        X = g.standard_normal((cols, B)).astype(np.float32)
+        enc = orc.encode(W, m)
+        Wd = _numpy_masked(enc)
+        exact = Wd @ X.astype(np.float64)
+        bound = (np.abs(Wd) @ np.abs(X.astype(np.float64))) * (cols + 1) * 2.0 ** -24
+        assert np.all(np.abs(orc.darb_spmm_f32(enc, X) - exact) <= bound)
+
+
 # --------------------------------------------------------------------------- RNN cells
 def _enc_rnn(orc, rows, cols, seed):
     g = np.random.default_rng(seed)
@@ -415,6 +437,6 @@ ALL_CHECKS = [
     check_assign_worked_example, check_assign_random, check_block_counts,
     check_pruning_ratio_identity, check_encode_random, check_encode_bf16,
     check_encode_special_values, check_encode_nan, check_product_exhaustive,
-    check_product_random, check_lstm_vs_torch, check_gru_vs_torch, check_rnn_zero_weights,
+    check_product_random, check_product_f32_timed, check_lstm_vs_torch, check_gru_vs_torch, check_rnn_zero_weights,
     check_gru_split_columns,
 ]
