@@ -31,6 +31,7 @@ struct darb_handle_s {
     std::vector<int32_t> rowmap, rowloc, row_m;
     std::vector<darb::EncTile> enc_tiles;   // every encoder tile, resolved
     int32_t max_tile = 0;                   // elements of the largest encoder tile (nb * m)
+    std::vector<darb::EncTile> row_tiles;   // tiles of the bf16 row encoder (empty where it does not apply)
     std::vector<darb::WorkItem> items;   // CTA work tables of every (level, split), concatenated
     int32_t item_first[darb::kWorkLevels][darb::kWorkSplits] = {};
     int32_t nitems[darb::kWorkLevels][darb::kWorkSplits] = {};
@@ -45,7 +46,7 @@ struct darb_handle_s {
     void *dmem = nullptr;
     size_t dbytes = 0;
     Group *d_groups = nullptr;
-    darb::EncTile *d_tiles = nullptr;
+    darb::EncTile *d_tiles = nullptr, *d_row_tiles = nullptr;
     darb::WorkItem *d_items = nullptr;
     int32_t *d_rowmap = nullptr, *d_rowloc = nullptr, *d_row_m = nullptr, *d_status = nullptr;
     void *d_vals = nullptr;
@@ -153,28 +154,38 @@ void build_layout(darb_handle_s *h, const int32_t *m) {
     h->val_elems = val;
     h->off_words = off;
     build_work_tables(h);
-    h->enc_tiles.clear();
-    h->max_tile = 0;
-    for (int64_t r = 0; r < rows; ++r) {
-        const int32_t loc = h->rowloc[static_cast<size_t>(r)];
-        const Group &g = h->groups[static_cast<size_t>(loc / kSlots)];
-        const int64_t slot = loc % kSlots;
-        const int tb = darb::enc_tile_blocks(g.m);
-        for (int64_t jt = 0; jt < g.n; jt += tb) {
-            darb::EncTile t{};
-            const int64_t nb = std::min<int64_t>(tb, g.n - jt);
-            const int64_t rec = (jt / kChunk) * kSlots + slot;   // jt is a multiple of the chunk
-            t.row = static_cast<int32_t>(r);
-            t.c0 = static_cast<int32_t>(jt * g.m);
-            t.span = static_cast<int32_t>(std::min<int64_t>(cols, (jt + nb) * g.m) - jt * g.m);
-            t.m = static_cast<int16_t>(g.m);
-            t.nb = static_cast<int16_t>(nb);
-            t.val_base = g.val_off + rec * kChunk;
-            t.off_base = g.off_off + rec * (g.nib ? 1 : 2);
-            h->enc_tiles.push_back(t);
-            h->max_tile = std::max<int32_t>(h->max_tile, static_cast<int32_t>(nb * g.m));
+    // tiles of tb(m) blocks, every row in order; tb a multiple of the chunk
+    auto tiles_of = [h, rows, cols](std::vector<darb::EncTile> &out, int (*tb_of)(int)) {
+        out.clear();
+        for (int64_t r = 0; r < rows; ++r) {
+            const int32_t loc = h->rowloc[static_cast<size_t>(r)];
+            const Group &g = h->groups[static_cast<size_t>(loc / kSlots)];
+            const int64_t slot = loc % kSlots;
+            const int tb = tb_of(g.m);
+            for (int64_t jt = 0; jt < g.n; jt += tb) {
+                darb::EncTile t{};
+                const int64_t nb = std::min<int64_t>(tb, g.n - jt);
+                const int64_t rec = (jt / kChunk) * kSlots + slot;   // jt is a multiple of the chunk
+                t.row = static_cast<int32_t>(r);
+                t.c0 = static_cast<int32_t>(jt * g.m);
+                t.span = static_cast<int32_t>(std::min<int64_t>(cols, (jt + nb) * g.m) - jt * g.m);
+                t.m = static_cast<int16_t>(g.m);
+                t.nb = static_cast<int16_t>(nb);
+                t.val_base = g.val_off + rec * kChunk;
+                t.off_base = g.off_off + rec * (g.nib ? 1 : 2);
+                out.push_back(t);
+            }
         }
-    }
+    };
+    tiles_of(h->enc_tiles, darb::enc_tile_blocks);
+    h->max_tile = 0;
+    for (const darb::EncTile &t : h->enc_tiles)
+        h->max_tile = std::max<int32_t>(h->max_tile, static_cast<int32_t>(t.nb) * t.m);
+    bool pow2 = h->wtype == DARB_BF16;
+    for (const Group &g : h->groups)
+        if (g.m < 8 || g.m > 256 || (g.m & (g.m - 1)) != 0) pow2 = false;
+    h->row_tiles.clear();
+    if (pow2) tiles_of(h->row_tiles, [](int m) { return darb::kRowPassElems / m; });
 }
 
 // The CTA work tables of batch_kernel (darb::WorkItem).  For row sets of up to
@@ -283,6 +294,7 @@ darb_status_t alloc_device(darb_handle_s *h) {
     size_t o = 0;
     const size_t o_groups = o; o = align_up(o + h->groups.size() * sizeof(Group), 256);
     const size_t o_tiles = o;  o = align_up(o + h->enc_tiles.size() * sizeof(darb::EncTile), 256);
+    const size_t o_rtiles = o; o = align_up(o + h->row_tiles.size() * sizeof(darb::EncTile), 256);
     const size_t o_items = o;  o = align_up(o + h->items.size() * sizeof(darb::WorkItem), 256);
     const size_t o_sgeo = o;   o = align_up(o + h->xsets.size() * sizeof(darb::SetGeo), 256);
     const size_t o_rowmap = o; o = align_up(o + h->rowmap.size() * 4, 256);
@@ -299,6 +311,7 @@ darb_status_t alloc_device(darb_handle_s *h) {
     h->dbytes = o;
     h->d_groups = reinterpret_cast<Group *>(b + o_groups);
     h->d_tiles = reinterpret_cast<darb::EncTile *>(b + o_tiles);
+    h->d_row_tiles = reinterpret_cast<darb::EncTile *>(b + o_rtiles);
     h->d_items = reinterpret_cast<darb::WorkItem *>(b + o_items);
     h->d_xsets = reinterpret_cast<darb::SetGeo *>(b + o_sgeo);
     h->d_rowmap = reinterpret_cast<int32_t *>(b + o_rowmap);
@@ -317,6 +330,9 @@ darb_status_t upload_layout(darb_handle_s *h, cudaStream_t stream) {
                             cudaMemcpyHostToDevice, stream);
     if (e == cudaSuccess)
         e = cudaMemcpyAsync(h->d_tiles, h->enc_tiles.data(), h->enc_tiles.size() * sizeof(darb::EncTile),
+                            cudaMemcpyHostToDevice, stream);
+    if (e == cudaSuccess && !h->row_tiles.empty())
+        e = cudaMemcpyAsync(h->d_row_tiles, h->row_tiles.data(), h->row_tiles.size() * sizeof(darb::EncTile),
                             cudaMemcpyHostToDevice, stream);
     if (e == cudaSuccess)
         e = cudaMemcpyAsync(h->d_items, h->items.data(), h->items.size() * sizeof(darb::WorkItem),
@@ -387,6 +403,8 @@ darb::EncodeTarget target_of(darb_handle_s *h) {
     t.tiles = h->d_tiles;
     t.ntiles = static_cast<int32_t>(h->enc_tiles.size());
     t.max_tile = h->max_tile;
+    t.row_tiles = h->d_row_tiles;
+    t.n_row_tiles = static_cast<int32_t>(h->row_tiles.size());
     t.vals = h->d_vals;
     t.offs = h->d_offs;
     t.bf16 = h->wtype == DARB_BF16 ? 1 : 0;

@@ -34,6 +34,10 @@ constexpr int kEncTileElems = 12288;   // columns of W the encoder stages per ti
 // blocks, a multiple of the chunk so that offset records never straddle tiles.
 inline __host__ __device__ int enc_tile_blocks(int m) { return (kEncTileElems / m) / kChunk * kChunk; }
 
+// The bf16 row encoder (block sizes powers of two from 8 to 256) takes tiles of
+// kRowPassElems columns: kRowPassElems / m blocks, a multiple of the chunk.
+constexpr int kRowPassElems = 2048;
+
 struct Group {
     int32_t m;        // block size shared by the group's rows
     int32_t n;        // blocks per row, ceil(cols / m)
@@ -129,6 +133,8 @@ struct EncodeTarget {
     const EncTile *tiles;    // every encoder tile, row-major
     int32_t ntiles;
     int32_t max_tile;        // elements of the largest tile, max over tiles of nb * m (zero padding included)
+    const EncTile *row_tiles;   // tiles of the bf16 row encoder (kRowPassElems columns), row-major
+    int32_t n_row_tiles;        // 0 unless the weights are bf16 and every block size a power of two in [8, 256]
     void *vals;
     uint32_t *offs;
     int32_t bf16;

@@ -55,11 +55,13 @@ __device__ __forceinline__ void mbar_expect_tx(uint64_t *bar, uint32_t bytes) {
 }
 
 // Wait for the phase with the given parity to complete; false after the time
-// limit.  Each try_wait may suspend the thread in hardware while the phase is
-// pending; with `backoff` the thread also sleeps between attempts (32 ns
-// doubling to 512 ns) so that a warp waiting long costs few issue slots,
-// without it the wait reacts as soon as the phase completes.
-__device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, bool backoff = true) {
+// limit.  Each try_wait suspends the thread in hardware while the phase is
+// pending (up to the hint), so polling costs few issue slots and the wait
+// ends as soon as the phase completes.  With `backoff` the thread also sleeps
+// between attempts (32 ns doubling to 512 ns); only for waits that are long
+// and not on a critical path: a thread that sleeps past the completion holds
+// up every thread that waits for it (a warp's shuffle, a CTA barrier).
+__device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, bool backoff = false) {
     const uint32_t a = smem_addr(bar);
     unsigned long long t0 = 0;
     unsigned sleep_ns = 32;
