@@ -26,6 +26,8 @@
 // group and x fit in shared memory and the arrays are 16-byte aligned.
 #pragma once
 
+#include <type_traits>
+
 #include "kernels_common.cuh"
 #include "launch.cuh"
 #include "tma.cuh"
@@ -35,13 +37,14 @@ namespace gemv {
 
 constexpr int kWarpsG = 16;
 constexpr int kThreadsG = kWarpsG * 32;
-// Chunks a lane has in flight at once.  Three keeps the kernel near 60
-// registers a thread: a CTA then fits beside the CTAs of the kernel before it
-// on the stream (the encoder's, say), so with PDL it starts its loads while
-// that kernel drains.  Four chunks run a lone launch ~15% faster but need ~84
-// registers, and the bench step (encode, then the products) came out ~3%
-// slower for it.
-constexpr int kBatchChunks = 3;
+// Chunks a lane has in flight at once (bf16 records).  Three keeps the kernel
+// near 60 registers a thread: a CTA then fits beside the CTAs of the kernel
+// before it on the stream (the encoder's, say), so with PDL it starts its
+// loads while that kernel drains.  Four chunks run a lone launch ~15% faster
+// but need ~84 registers, and the bench step (encode, then the products) came
+// out ~3% slower for it.  fp32 records are twice the size: two chunks.
+template <bool BF16>
+__host__ __device__ constexpr int batch_chunks() { return BF16 ? 3 : 2; }
 constexpr size_t kMaxCols = 48 * 1024;   // x in shared memory: 192 KB at most
 
 template <bool BF16>
@@ -64,34 +67,69 @@ __device__ __forceinline__ void load_chunk_rec(const Format &f, const Group &g, 
     else d.o = __ldg(reinterpret_cast<const uint2 *>(f.offs + g.off_off) + rec);
 }
 
-template <bool BF16>
-__device__ __forceinline__ float chunk_dot(const Group &g, int c, const ChunkData<BF16> &d, const float *s_x) {
-    float v[kChunk];
-    if constexpr (BF16) {
-        const uint32_t w[4] = {d.v[0].x, d.v[0].y, d.v[0].z, d.v[0].w};
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-            v[2 * e] = __uint_as_float(w[e] << 16);
-            v[2 * e + 1] = __uint_as_float(w[e] & 0xFFFF0000u);
-        }
-    } else {
-        v[0] = __uint_as_float(d.v[0].x); v[1] = __uint_as_float(d.v[0].y);
-        v[2] = __uint_as_float(d.v[0].z); v[3] = __uint_as_float(d.v[0].w);
-        v[4] = __uint_as_float(d.v[1].x); v[5] = __uint_as_float(d.v[1].y);
-        v[6] = __uint_as_float(d.v[1].z); v[7] = __uint_as_float(d.v[1].w);
-    }
-    const int m = g.m, n = g.n;
-    const bool full = (c + 1) * kChunk <= n;
-    float acc = 0.0f;
+// A chunk's products for one slot (lane): block e selects xb[e m + offset],
+// xb = x + 8 c m.  The offset width and, for every chunk but a row's last, the
+// 8 blocks' existence are known at compile time, so an element costs an
+// extract, an address, a gather and an FMA; two accumulators (even and odd
+// blocks) keep independent gathers in flight.
+template <bool BF16, bool NIB, bool FULL>
+__device__ __forceinline__ float chunk_sum(const ChunkData<BF16> &d, const float *xb, int m, int nvalid) {
+    float a0 = 0.0f, a1 = 0.0f;
 #pragma unroll
     for (int e = 0; e < kChunk; ++e) {
-        const int j = c * kChunk + e;
-        if (full || j < n) {
-            const uint32_t o = g.nib ? (d.o.x >> (4 * e)) & 15u : ((e < 4 ? d.o.x : d.o.y) >> (8 * (e & 3))) & 255u;
-            acc = fmaf(v[e], s_x[j * m + int(o)], acc);
+        if (FULL || e < nvalid) {
+            const uint32_t o = NIB ? (d.o.x >> (4 * e)) & 15u : ((e < 4 ? d.o.x : d.o.y) >> (8 * (e & 3))) & 255u;
+            const uint4 &q = d.v[BF16 ? 0 : e >> 2];
+            const uint32_t word = BF16 ? ((e >> 1) == 0 ? q.x : (e >> 1) == 1 ? q.y : (e >> 1) == 2 ? q.z : q.w)
+                                       : ((e & 3) == 0 ? q.x : (e & 3) == 1 ? q.y : (e & 3) == 2 ? q.z : q.w);
+            const float v = BF16 ? __uint_as_float((e & 1) ? (word & 0xFFFF0000u) : (word << 16)) : __uint_as_float(word);
+            const float x = xb[e * m + int(o)];
+            if ((e & 1) && BF16) a1 = fmaf(v, x, a1);   // fp32 records: one chain (register pressure)
+            else a0 = fmaf(v, x, a0);
         }
     }
-    return acc;
+    return a0 + a1;
+}
+
+// Chunk c's products for one slot: a row's last chunk may hold fewer than 8 blocks.
+template <bool BF16, bool NIB>
+__device__ __forceinline__ float chunk_at(const ChunkData<BF16> &d, int c, int n, int m, const float *xs) {
+    const float *xb = xs + c * kChunk * m;
+    return (c + 1) * kChunk <= n ? chunk_sum<BF16, NIB, true>(d, xb, m, kChunk)
+                                 : chunk_sum<BF16, NIB, false>(d, xb, m, n - c * kChunk);
+}
+
+// The record of chunk `rec` (lane = slot) from the shared-memory copies of a
+// group's values and offsets.
+template <bool BF16, bool NIB>
+__device__ __forceinline__ ChunkData<BF16> smem_chunk(const unsigned char *s_val, const uint32_t *s_off, int rec) {
+    ChunkData<BF16> d;
+    if constexpr (BF16) {
+        d.v[0] = reinterpret_cast<const uint4 *>(s_val)[rec];
+    } else {
+        d.v[0] = reinterpret_cast<const uint4 *>(s_val)[2 * rec];
+        d.v[1] = reinterpret_cast<const uint4 *>(s_val)[2 * rec + 1];
+    }
+    d.o = NIB ? make_uint2(s_off[rec], 0u) : reinterpret_cast<const uint2 *>(s_off)[rec];
+    return d;
+}
+
+// Warp `warp`'s share of a group held in shared memory: chunks warp, warp +
+// WARPS, ..., two at a time.
+template <bool BF16, bool NIB, int WARPS>
+__device__ __forceinline__ float group_sum(const unsigned char *s_val, const uint32_t *s_off, const float *xs,
+                                           int nch, int n, int m, int warp, int lane) {
+    float acc0 = 0.0f, acc1 = 0.0f;
+    int c = warp;
+    auto one = [&](int cc, float &acc) {
+        acc += chunk_at<BF16, NIB>(smem_chunk<BF16, NIB>(s_val, s_off, cc * kSlots + lane), cc, n, m, xs);
+    };
+    for (; c + WARPS < nch; c += 2 * WARPS) {
+        one(c, acc0);
+        one(c + WARPS, acc1);
+    }
+    if (c < nch) one(c, acc0);
+    return acc0 + acc1;
 }
 
 template <bool BF16>
@@ -107,11 +145,11 @@ gemv_kernel(Format f, const float *X, int64_t ldx, float *Y, int64_t ldy, int ea
     pdl_launch_dependents();
     // the first batch of this warp's chunks: the handle's data never changes
     // after encoding, so with `early` it is read before the previous kernel ends
-    ChunkData<BF16> d[kBatchChunks];
+    ChunkData<BF16> d[batch_chunks<BF16>()];
     int c0 = warp;
     auto load_batch = [&](int cfirst) {
 #pragma unroll
-        for (int k = 0; k < kBatchChunks; ++k) {
+        for (int k = 0; k < batch_chunks<BF16>(); ++k) {
             const int c = cfirst + k * kWarpsG;
             if (c < nch) load_chunk_rec<BF16>(f, g, c, lane, d[k]);
         }
@@ -131,15 +169,20 @@ gemv_kernel(Format f, const float *X, int64_t ldx, float *Y, int64_t ldy, int ea
     }
     __syncthreads();
     float acc = 0.0f;
-    while (c0 < nch) {
+    auto run = [&](auto nib) {   // the offset width fixed for the whole loop
+        constexpr bool NIB = decltype(nib)::value;
+        while (c0 < nch) {
 #pragma unroll
-        for (int k = 0; k < kBatchChunks; ++k) {
-            const int c = c0 + k * kWarpsG;
-            if (c < nch) acc += chunk_dot<BF16>(g, c, d[k], s_x);
+            for (int k = 0; k < batch_chunks<BF16>(); ++k) {
+                const int c = c0 + k * kWarpsG;
+                if (c < nch) acc += chunk_at<BF16, NIB>(d[k], c, g.n, g.m, s_x);
+            }
+            c0 += batch_chunks<BF16>() * kWarpsG;
+            if (c0 < nch) load_batch(c0);
         }
-        c0 += kBatchChunks * kWarpsG;
-        if (c0 < nch) load_batch(c0);
-    }
+    };
+    if (g.nib) run(std::true_type{});
+    else run(std::false_type{});
     s_part[warp][lane] = acc;
     __syncthreads();
     if (warp == 0 && lane < g.nrows) {
@@ -150,10 +193,15 @@ gemv_kernel(Format f, const float *X, int64_t ldx, float *Y, int64_t ldy, int ea
     }
 }
 
+// Warps of gemv_bulk_kernel (32 split a group's chunks twice as finely but ran
+// FC6 at batch 1 in 3.4 us against 3.2 for 16).
+constexpr int kWarpsB = 16;
+constexpr int kThreadsB = kWarpsB * 32;
+
 // Shared memory of gemv_bulk_kernel: [0, 128) the two mbarriers, then vcap
 // bytes for a group's values, ocap for its offsets, then x.
 template <bool BF16>
-__global__ void __launch_bounds__(kThreadsG)
+__global__ void __launch_bounds__(kThreadsB)
 gemv_bulk_kernel(Format f, const float *X, int64_t ldx, float *Y, int64_t ldy, int early, int vcap, int ocap) {
     constexpr int kEsz = BF16 ? 2 : 4;
     extern __shared__ __align__(128) unsigned char sm[];
@@ -161,7 +209,7 @@ gemv_bulk_kernel(Format f, const float *X, int64_t ldx, float *Y, int64_t ldy, i
     unsigned char *const s_val = sm + 128;
     uint32_t *const s_off = reinterpret_cast<uint32_t *>(s_val + vcap);
     float *const s_x = reinterpret_cast<float *>(reinterpret_cast<unsigned char *>(s_off) + ocap);
-    __shared__ float s_part[kWarpsG][kSlots];
+    __shared__ float s_part[kWarpsB][kSlots];
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int gi = blockIdx.x;
     const Group g = f.groups[gi];
@@ -193,23 +241,13 @@ gemv_bulk_kernel(Format f, const float *X, int64_t ldx, float *Y, int64_t ldy, i
         }
     }
     if (!xbulk)
-        for (int64_t k = tid; k < cols; k += kThreadsG) s_x[k] = __ldg(X + k * ldx);
+        for (int64_t k = tid; k < cols; k += kThreadsB) s_x[k] = __ldg(X + k * ldx);
     __syncthreads();   // the barriers' initialisation and the plain copy of x are seen by all threads
     const bool ok = __syncthreads_and(mbar_wait(&bar[0], 0) && (!xbulk || mbar_wait(&bar[1], 0)));
     float acc = 0.0f;
     if (ok) {
-        for (int c = warp; c < nch; c += kWarpsG) {
-            const int rec = c * kSlots + lane;
-            ChunkData<BF16> d;
-            if constexpr (BF16) {
-                d.v[0] = reinterpret_cast<const uint4 *>(s_val)[rec];
-            } else {
-                d.v[0] = reinterpret_cast<const uint4 *>(s_val)[2 * rec];
-                d.v[1] = reinterpret_cast<const uint4 *>(s_val)[2 * rec + 1];
-            }
-            d.o = g.nib ? make_uint2(s_off[rec], 0u) : reinterpret_cast<const uint2 *>(s_off)[rec];
-            acc += chunk_dot<BF16>(g, c, d, s_x);
-        }
+        acc = g.nib ? group_sum<BF16, true, kWarpsB>(s_val, s_off, s_x, nch, g.n, g.m, warp, lane)
+                    : group_sum<BF16, false, kWarpsB>(s_val, s_off, s_x, nch, g.n, g.m, warp, lane);
     } else if (tid == 0) {
         // a copy did not land in time: record it, and give the copies still in
         // flight a second bounded wait before the CTA (and its shared memory) ends
@@ -222,7 +260,7 @@ gemv_bulk_kernel(Format f, const float *X, int64_t ldx, float *Y, int64_t ldy, i
     if (ok && warp == 0 && lane < g.nrows) {
         float sum = 0.0f;
 #pragma unroll
-        for (int w = 0; w < kWarpsG; ++w) sum += s_part[w][lane];
+        for (int w = 0; w < kWarpsB; ++w) sum += s_part[w][lane];
         Y[int64_t(f.rowmap[gi * kSlots + lane]) * ldy] = sum;
     }
 }
@@ -233,8 +271,8 @@ template <bool BF16>
 cudaError_t launch(const Format &f, const float *X, int64_t ldx, float *Y, int64_t ldy, bool early,
                    cudaStream_t stream) {
     // the largest group is one of the smallest block size
-    if (f.m_min > 0 && (reinterpret_cast<uintptr_t>(f.vals) & 15) == 0 &&
-        (reinterpret_cast<uintptr_t>(f.offs) & 15) == 0) {
+    const bool aligned = (reinterpret_cast<uintptr_t>(f.vals) & 15) == 0 && (reinterpret_cast<uintptr_t>(f.offs) & 15) == 0;
+    if (f.m_min > 0 && aligned) {
         const int64_t nch = ((f.cols + f.m_min - 1) / f.m_min + kChunk - 1) / kChunk;
         const int64_t vcap = nch * kSlots * kChunk * (BF16 ? 2 : 4);
         // any group (m >= m_min) has at most nch chunks; room for 8-byte offset
@@ -244,7 +282,7 @@ cudaError_t launch(const Format &f, const float *X, int64_t ldx, float *Y, int64
         if (smem <= int64_t(kBulkSmemLimit)) {
             const cudaError_t attr = allow_smem(gemv_bulk_kernel<BF16>, kBulkSmemLimit);
             if (attr != cudaSuccess) return attr;
-            return launch_ex(gemv_bulk_kernel<BF16>, dim3(static_cast<unsigned>(f.ngroups)), dim3(kThreadsG),
+            return launch_ex(gemv_bulk_kernel<BF16>, dim3(static_cast<unsigned>(f.ngroups)), dim3(kThreadsB),
                              size_t(smem), stream, 1, true, f, X, ldx, Y, ldy, early ? 1 : 0, int(vcap), int(ocap));
         }
     }
