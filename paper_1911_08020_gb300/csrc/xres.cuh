@@ -19,10 +19,12 @@
 //    fixed number of groups of the heaviest bin (the SetGeo tables of the
 //    handle); units in tile-major order; each cluster takes a contiguous run
 //    of units of about equal work, so it loads the tile of a run once or twice;
-//  * 16 consumer warps: T/4 lanes per row, each lane 4 columns (one 16-byte
-//    load per kept weight; a quarter-warp reads 64 or 128 contiguous bytes of
-//    one activation row); a thread owns 1 to 4 rows of the set and works on
-//    the same chunk of all of them at once, so their loads overlap;
+//  * 16 consumer warps: 4 lanes per row, each lane 8 of the tile's 32
+//    columns (two 16-byte loads per kept weight, so that one offset, one value
+//    and one address serve 8 FMAs; the two rows of a quarter-warp read
+//    opposite halves of their activation rows, which keeps the loads free of
+//    bank conflicts); a pass covers 128 rows, a thread owns 1 or 2 rows of the
+//    set;
 //  * one producer warp: bulk copies of the values and offsets of each round
 //    (a run of chunks of the set's groups) into a 6-stage ring with full /
 //    empty mbarriers, and tensor-map copies of the tile slice (rows past the
@@ -66,6 +68,15 @@ namespace xres {
 
 namespace cg = cooperative_groups;
 
+// 16 bytes of the staged activation slice at a 32-bit shared address.  Not
+// volatile: the address depends on offsets read after the stage's wait, and
+// the slice itself changes only across a wait on xfull.
+__device__ __forceinline__ float4 lds_f4(uint32_t addr) {
+    float4 v;
+    asm("ld.shared.v4.f32 {%0, %1, %2, %3}, [%4];" : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w) : "r"(addr));
+    return v;
+}
+
 constexpr int kCWarps = 16;                    // consumer warps
 constexpr int kCThreads = kCWarps * 32;
 constexpr int kRWarps = 3;                     // reducer warps (20 warps in all: 96 registers a thread)
@@ -86,10 +97,6 @@ template <bool BF16>
 __host__ __device__ constexpr uint32_t ring_val_bytes() { return kRecCap * rec_val_bytes<BF16>(); }
 template <bool BF16>
 __host__ __device__ constexpr uint32_t stage_bytes() { return ring_val_bytes<BF16>() + kRecCap * kRecOffBytes; }
-
-// Rows one pass of the consumers covers: T/4 lanes per row.
-template <int T>
-__host__ __device__ constexpr int pass_rows() { return kCWarps * 32 / (T / 4); }
 
 struct Plan {
     int C;            // CTAs per cluster = column slices
@@ -121,9 +128,7 @@ template <bool BF16, int T>
 __global__ void __launch_bounds__(kThreads, 1)
 xres_kernel(Format f, const float *__restrict__ X, int64_t batch, float *__restrict__ Y, int64_t ldy,
             const __grid_constant__ CUtensorMap xmap, const __grid_constant__ Plan p) {
-    constexpr int kLpr = T / 4;             // lanes per row
-    constexpr int kRpw = 32 / kLpr;         // rows per warp and pass
-    constexpr int kPassRows = pass_rows<T>();
+    static_assert(T == 32, "the consumer layouts assume 32-column tiles (128-byte activation rows)");
     constexpr int kEsz = BF16 ? 2 : 4;
     extern __shared__ __align__(128) unsigned char sm[];
     Bars &bar = *reinterpret_cast<Bars *>(sm);
@@ -336,26 +341,39 @@ xres_kernel(Format f, const float *__restrict__ X, int64_t batch, float *__restr
         if (!ok && lane == 0) atomicOr(f.status, kStatusTimeout);
     } else {
         // ------------------------------------------------------------ consumers
-        const int qd = lane % kLpr;                 // float4 of the tile this lane owns
-        const int rs = warp * kRpw + lane / kLpr;   // row of the set in pass 0
+        // Two layouts of the consumer threads, chosen per set:
+        //  * LPR = 4 lanes a row (sets of more than 64 rows): a lane owns 8 of
+        //    the tile's 32 columns, quads qd + 4h and then qd + 4(1 - h) (h =
+        //    parity of its row), so that one offset, one value and one address
+        //    serve two 16-byte loads, and the two rows of a quarter-warp read
+        //    opposite halves of their activation rows -- 8 distinct bank groups;
+        //  * LPR = 8 lanes a row (sets of up to 64 rows, which would leave half
+        //    of a 128-row pass idle): a lane owns one quad, a quarter-warp reads
+        //    one whole activation row.
         bool ok = true;
         int rc = 0, xloads = 0, cur_tile = -1;
         Cursor cu = cursor_at(u_begin), cn = cu;
         advance(cn);
         Set s_next = u_begin < u_end ? load_set(cu.sidx) : Set{};
-        // this lane's 16 bytes of row 0 of the slice
-        const unsigned char *xl = reinterpret_cast<const unsigned char *>(s_x) + qd * 16;
-        constexpr int kRowShift = T == 32 ? 7 : 6;   // bytes of a staged activation row, log2
-        // one unit with NP row passes and 4-bit (NIB) or 8-bit offsets:
-        // multiply, then store the partial sums once every CTA's reducers
-        // have read the previous set's (t: sets stored)
-        auto unit = [&](auto npc, auto nibc, const Set &s, const Unit &g, int t) {
+        const uint32_t x0 = smem_addr(s_x);   // slice row k at x0 + 128 k (rows of 32 floats)
+        // one unit with LPR lanes a row, NP row passes and 4-bit (NIB) or 8-bit
+        // offsets: multiply, then store the partial sums once every CTA's
+        // reducers have read the previous set's (t: sets stored)
+        auto unit = [&](auto lprc, auto npc, auto nibc, const Set &s, const Unit &g, int t) {
+            constexpr int LPR = decltype(lprc)::value;
             constexpr int NP = decltype(npc)::value;
             constexpr bool NIB = decltype(nibc)::value;
-            float4 acc[NP];
+            constexpr bool kTwo = LPR == 4;          // two quads a lane
+            constexpr int kRpw = 32 / LPR;           // rows per warp and pass
+            constexpr int kPassRows = kCWarps * kRpw;
+            const int qd = lane % LPR;
+            const int cA = kTwo ? qd + 4 * ((lane >> 2) & 1) : qd;   // the lane's (first) column quad
+            const int cB = cA ^ 4;                                   // its second (LPR = 4)
+            const int rs = warp * kRpw + lane / LPR;                 // row of the set in pass 0
+            const uint32_t xl = x0 + uint32_t(cA) * 16u;
+            float4 accA[NP], accB[NP];
 #pragma unroll
-            for (int pp = 0; pp < NP; ++pp) acc[pp] = make_float4(0.f, 0.f, 0.f, 0.f);
-            float4 acc2 = make_float4(0.f, 0.f, 0.f, 0.f);   // odd chunks of a chunk pair (NP == 1)
+            for (int pp = 0; pp < NP; ++pp) accA[pp] = accB[pp] = make_float4(0.f, 0.f, 0.f, 0.f);
             // a row past the set (the last pass of a set with fewer groups) repeats a
             // row of its last group; its sums are stored but never read
             int gip[NP], slotp[NP];
@@ -365,7 +383,7 @@ xres_kernel(Format f, const float *__restrict__ X, int64_t batch, float *__restr
                 gip[pp] = min(row / kSlots, s.ng - 1);
                 slotp[pp] = row % kSlots;
             }
-            const int mrow = s.m << kRowShift;   // bytes between the first rows of consecutive blocks
+            const uint32_t mrow = uint32_t(s.m) << 7;   // bytes between the first rows of consecutive blocks
             for (int r = 0; r < g.rounds; ++r, ++rc) {
                 const int st = rc % kStages;
                 if (ok) ok = mbar_wait(&bar.full[st], (rc / kStages) & 1, false);
@@ -374,129 +392,62 @@ xres_kernel(Format f, const float *__restrict__ X, int64_t batch, float *__restr
                     const int cr0 = g.c0 + r * g.cpr, nchr = min(g.cpr, g.nch - r * g.cpr);
                     const unsigned char *sv = s_ring + size_t(st) * stage_bytes<BF16>();
                     const uint32_t *so = reinterpret_cast<const uint32_t *>(sv + ring_val_bytes<BF16>());
-                    int lc = 0;
-                    if constexpr (NP == 1) {
-                        // one row a thread: two whole chunks at a time, into two
-                        // accumulators, so that 16 gathers are in flight and the
-                        // records of both chunks load together
-                        const int slot0 = slotp[0], gi0 = gip[0];
-                        for (; lc + 1 < nchr; lc += 2) {
-                            const int jc = (cr0 + lc) * kChunk;
-                            if (jc < g.j0 || jc + 2 * kChunk > g.j1) break;   // not two whole chunks
-                            const int rec0 = (gi0 * nchr + lc) * kSlots + slot0, rec1 = rec0 + kSlots;
-                            uint32_t va[BF16 ? 4 : 8], vb[BF16 ? 4 : 8];
-                            uint2 oa, ob;
-                            {
-                                const uint4 *pa = reinterpret_cast<const uint4 *>(sv) + rec0 * (BF16 ? 1 : 2);
-                                const uint4 *pb = reinterpret_cast<const uint4 *>(sv) + rec1 * (BF16 ? 1 : 2);
-                                const uint4 a0 = pa[0], b0 = pb[0];
-                                va[0] = a0.x; va[1] = a0.y; va[2] = a0.z; va[3] = a0.w;
-                                vb[0] = b0.x; vb[1] = b0.y; vb[2] = b0.z; vb[3] = b0.w;
-                                if constexpr (!BF16) {
-                                    const uint4 a1 = pa[1], b1 = pb[1];
-                                    va[4] = a1.x; va[5] = a1.y; va[6] = a1.z; va[7] = a1.w;
-                                    vb[4] = b1.x; vb[5] = b1.y; vb[6] = b1.z; vb[7] = b1.w;
-                                }
-                                if constexpr (NIB) {
-                                    oa = make_uint2(so[rec0], 0u);
-                                    ob = make_uint2(so[rec1], 0u);
-                                } else {
-                                    oa = reinterpret_cast<const uint2 *>(so)[rec0];
-                                    ob = reinterpret_cast<const uint2 *>(so)[rec1];
-                                }
-                            }
-                            const int xa = (jc * s.m - kq0) << kRowShift, xbb = xa + (s.m << (kRowShift + 3));
-                            float4 &a = acc[0];
-                            float4 &b = acc2;
-#pragma unroll
-                            for (int e = 0; e < kChunk; ++e) {
-                                int offa, offb;
-                                if constexpr (NIB) {
-                                    offa = int((oa.x >> (4 * e)) & 15u);
-                                    offb = int((ob.x >> (4 * e)) & 15u);
-                                } else {
-                                    offa = int(((e < 4 ? oa.x : oa.y) >> (8 * (e & 3))) & 255u);
-                                    offb = int(((e < 4 ? ob.x : ob.y) >> (8 * (e & 3))) & 255u);
-                                }
-                                float wa, wb;
-                                if constexpr (BF16) {
-                                    wa = __uint_as_float((e & 1) ? (va[e >> 1] & 0xFFFF0000u) : (va[e >> 1] << 16));
-                                    wb = __uint_as_float((e & 1) ? (vb[e >> 1] & 0xFFFF0000u) : (vb[e >> 1] << 16));
-                                } else {
-                                    wa = __uint_as_float(va[e]);
-                                    wb = __uint_as_float(vb[e]);
-                                }
-                                const float4 x0 = *reinterpret_cast<const float4 *>(xl + (xa + e * mrow + (offa << kRowShift)));
-                                const float4 x1 = *reinterpret_cast<const float4 *>(xl + (xbb + e * mrow + (offb << kRowShift)));
-                                a.x = fmaf(wa, x0.x, a.x);
-                                a.y = fmaf(wa, x0.y, a.y);
-                                a.z = fmaf(wa, x0.z, a.z);
-                                a.w = fmaf(wa, x0.w, a.w);
-                                b.x = fmaf(wb, x1.x, b.x);
-                                b.y = fmaf(wb, x1.y, b.y);
-                                b.z = fmaf(wb, x1.z, b.z);
-                                b.w = fmaf(wb, x1.w, b.w);
-                            }
-                        }
-                    }
-                    for (; lc < nchr; ++lc) {
+                    for (int lc = 0; lc < nchr; ++lc) {
                         const int jc = (cr0 + lc) * kChunk;
                         const int e_lo = max(0, g.j0 - jc), e_hi = min(kChunk, g.j1 - jc);
-                        // byte offset of the slice row selected by block jc + e:
-                        // ((jc + e) * m + off - kq0) << kRowShift (xb is negative for a first
+                        // address of the slice row selected by block jc + e:
+                        // xl + (((jc + e) * m + off - kq0) << 7) (below the slice for a first
                         // chunk whose leading blocks belong to the previous slice; those
                         // blocks are never read)
-                        const int xb = (jc * s.m - kq0) << kRowShift;
-                        // rows in sub-groups of kSub, so that their values, offsets and
-                        // loads in flight fit in registers
-                        constexpr int kSub = NP < 2 ? NP : 2;
+                        const uint32_t xb = xl + (uint32_t(jc * s.m - kq0) << 7);
 #pragma unroll
-                        for (int p0 = 0; p0 < NP; p0 += kSub) {
-                            uint32_t vw[kSub][BF16 ? 4 : 8];
-                            uint2 ow[kSub];
-#pragma unroll
-                            for (int k = 0; k < kSub; ++k) {
-                                const int rec = (gip[p0 + k] * nchr + lc) * kSlots + slotp[p0 + k];
+                        for (int pp = 0; pp < NP; ++pp) {
+                            const int rec = (gip[pp] * nchr + lc) * kSlots + slotp[pp];
+                            uint32_t vw[BF16 ? 4 : 8];
+                            {
                                 const uint4 *pv = reinterpret_cast<const uint4 *>(sv) + rec * (BF16 ? 1 : 2);
                                 const uint4 w0 = pv[0];
-                                vw[k][0] = w0.x; vw[k][1] = w0.y; vw[k][2] = w0.z; vw[k][3] = w0.w;
+                                vw[0] = w0.x; vw[1] = w0.y; vw[2] = w0.z; vw[3] = w0.w;
                                 if constexpr (!BF16) {
                                     const uint4 w1 = pv[1];
-                                    vw[k][4] = w1.x; vw[k][5] = w1.y; vw[k][6] = w1.z; vw[k][7] = w1.w;
+                                    vw[4] = w1.x; vw[5] = w1.y; vw[6] = w1.z; vw[7] = w1.w;
                                 }
-                                if constexpr (NIB) ow[k] = make_uint2(so[rec], 0u);
-                                else ow[k] = reinterpret_cast<const uint2 *>(so)[rec];
                             }
-                            // block e of row p0 + k: its kept value times its selected activation row
-                            auto block = [&](int e, int k) {
-                                int off;
-                                if constexpr (NIB) off = int((ow[k].x >> (4 * e)) & 15u);
-                                else off = int(((e < 4 ? ow[k].x : ow[k].y) >> (8 * (e & 3))) & 255u);
+                            const uint2 ow = NIB ? make_uint2(so[rec], 0u) : reinterpret_cast<const uint2 *>(so)[rec];
+                            // block e: its kept value times the lane's quads of its selected activation row
+                            auto block = [&](int e) {
+                                uint32_t off;
+                                if constexpr (NIB) off = (ow.x >> (4 * e)) & 15u;
+                                else off = ((e < 4 ? ow.x : ow.y) >> (8 * (e & 3))) & 255u;
                                 float v;
                                 if constexpr (BF16)
-                                    v = __uint_as_float((e & 1) ? (vw[k][e >> 1] & 0xFFFF0000u) : (vw[k][e >> 1] << 16));
+                                    v = __uint_as_float((e & 1) ? (vw[e >> 1] & 0xFFFF0000u) : (vw[e >> 1] << 16));
                                 else
-                                    v = __uint_as_float(vw[k][e]);
-                                const float4 xv =
-                                    *reinterpret_cast<const float4 *>(xl + (xb + e * mrow + (off << kRowShift)));
-                                float4 &a = acc[p0 + k];
-                                a.x = fmaf(v, xv.x, a.x);
-                                a.y = fmaf(v, xv.y, a.y);
-                                a.z = fmaf(v, xv.z, a.z);
-                                a.w = fmaf(v, xv.w, a.w);
+                                    v = __uint_as_float(vw[e]);
+                                const uint32_t ad = xb + uint32_t(e) * mrow + (off << 7);
+                                const float4 xa = lds_f4(ad);
+                                float4 &a = accA[pp];
+                                a.x = fmaf(v, xa.x, a.x);
+                                a.y = fmaf(v, xa.y, a.y);
+                                a.z = fmaf(v, xa.z, a.z);
+                                a.w = fmaf(v, xa.w, a.w);
+                                if constexpr (kTwo) {
+                                    const float4 xc = lds_f4(ad ^ 64u);   // the other half of the row
+                                    float4 &b = accB[pp];
+                                    b.x = fmaf(v, xc.x, b.x);
+                                    b.y = fmaf(v, xc.y, b.y);
+                                    b.z = fmaf(v, xc.z, b.z);
+                                    b.w = fmaf(v, xc.w, b.w);
+                                }
                             };
                             if (e_lo == 0 && e_hi == kChunk) {
                                 // a whole chunk: one straight run, every load can be issued early
 #pragma unroll
-                                for (int e = 0; e < kChunk; ++e)
-#pragma unroll
-                                    for (int k = 0; k < kSub; ++k) block(e, k);
+                                for (int e = 0; e < kChunk; ++e) block(e);
                             } else {
 #pragma unroll
                                 for (int e = 0; e < kChunk; ++e)
-                                    if (e >= e_lo && e < e_hi)
-#pragma unroll
-                                        for (int k = 0; k < kSub; ++k) block(e, k);
+                                    if (e >= e_lo && e < e_hi) block(e);
                             }
                         }
                     }
@@ -504,16 +455,13 @@ xres_kernel(Format f, const float *__restrict__ X, int64_t batch, float *__restr
                 __syncwarp();
                 if (lane == 0) mbar_arrive(&bar.empty[st]);
             }
-            if constexpr (NP == 1) {   // the two chunk streams, in a fixed order
-                acc[0].x += acc2.x;
-                acc[0].y += acc2.y;
-                acc[0].z += acc2.z;
-                acc[0].w += acc2.w;
-            }
             if (t >= 1 && ok) ok = mbar_wait_acq_cluster(&bar.freed, (t - 1) & 1);
 #pragma unroll
-            for (int pp = 0; pp < NP; ++pp)
-                reinterpret_cast<float4 *>(s_part)[(rs + pp * kPassRows) * kLpr + qd] = acc[pp];
+            for (int pp = 0; pp < NP; ++pp) {
+                float4 *pr = reinterpret_cast<float4 *>(s_part) + (rs + pp * kPassRows) * (T / 4);
+                pr[cA] = accA[pp];
+                if constexpr (kTwo) pr[cB] = accB[pp];
+            }
         };
         int t = 0;   // sets stored
         for (int u = u_begin; u < u_end; ++u, ++t, cu = cn, advance(cn)) {
@@ -530,21 +478,23 @@ xres_kernel(Format f, const float *__restrict__ X, int64_t batch, float *__restr
                 ++xloads;
                 cur_tile = g.tile;
             }
-            const int np = (s.ng * kSlots + kPassRows - 1) / kPassRows;
+            using L4 = std::integral_constant<int, 4>;
+            using L8 = std::integral_constant<int, 8>;
             using N1 = std::integral_constant<int, 1>;
             using N2 = std::integral_constant<int, 2>;
-            using N4 = std::integral_constant<int, 4>;
             using Nib = std::true_type;
             using Byte = std::false_type;
-            if (np <= 1) {
-                if (s.nib) unit(N1{}, Nib{}, s, g, t);
-                else unit(N1{}, Byte{}, s, g, t);
-            } else if (np == 2) {
-                if (s.nib) unit(N2{}, Nib{}, s, g, t);
-                else unit(N2{}, Byte{}, s, g, t);
-            } else if constexpr (4 * kPassRows <= kMaxGroups * kSlots) {
-                if (s.nib) unit(N4{}, Nib{}, s, g, t);
-                else unit(N4{}, Byte{}, s, g, t);
+            static_assert(2 * kCWarps * 8 >= kMaxGroups * kSlots, "two 128-row passes cover the largest set");
+            const int rows = s.ng * kSlots;
+            if (rows <= kCWarps * 4) {          // one pass of 8 lanes a row
+                if (s.nib) unit(L8{}, N1{}, Nib{}, s, g, t);
+                else unit(L8{}, N1{}, Byte{}, s, g, t);
+            } else if (rows <= kCWarps * 8) {   // one pass of 4 lanes a row
+                if (s.nib) unit(L4{}, N1{}, Nib{}, s, g, t);
+                else unit(L4{}, N1{}, Byte{}, s, g, t);
+            } else {
+                if (s.nib) unit(L4{}, N2{}, Nib{}, s, g, t);
+                else unit(L4{}, N2{}, Byte{}, s, g, t);
             }
             // this warp's partial sums are stored: tell every CTA's reducers
             __syncwarp();
@@ -594,11 +544,10 @@ template <bool BF16, int T>
 cudaError_t launch(const Format &f, const float *X, int64_t ldx, int64_t batch, float *Y, int64_t ldy, bool early,
                    cudaStream_t stream) {
     (void)early;
-    const int table = T == 32 ? 0 : 1;   // sets of about 2 (T = 32) or 4 (T = 16) heaviest groups
-    const int nsets = f.nxsets[table];
     const int64_t tiles = (batch + T - 1) / T;
-    const int64_t units = tiles * nsets;
-    if (nsets <= 0 || units > (int64_t(1) << 30) || f.xset_prefix[table] == nullptr) return cudaErrorNotSupported;
+    if (f.nxsets[0] <= 0 || f.nxsets[1] <= 0 || f.xset_prefix[0] == nullptr || f.xset_prefix[1] == nullptr ||
+        tiles * f.nxsets[0] > (int64_t(1) << 30))
+        return cudaErrorNotSupported;
     if (reinterpret_cast<uintptr_t>(X) % 16 != 0 || (ldx * 4) % 16 != 0) return cudaErrorNotSupported;
     PFN_cuTensorMapEncodeTiled_v12000 enc = tensor_map_encoder();
     if (enc == nullptr) return cudaErrorNotSupported;
@@ -612,7 +561,6 @@ cudaError_t launch(const Format &f, const float *X, int64_t ldx, int64_t batch, 
         const int64_t rows = std::min<int64_t>(f.cols, S + f.m_max - 1);
         const int nboxes = static_cast<int>((rows + 255) / 256);
         int box_rows = static_cast<int>((rows + nboxes - 1) / nboxes);
-        if (T == 16) box_rows = (box_rows + 1) & ~1;   // every box lands on a 128-byte boundary
         const uint64_t x_bytes = uint64_t(nboxes) * box_rows * T * 4;
         const uint64_t ring_off = 128 + x_bytes;
         const uint64_t part_off = ring_off + uint64_t(kStages) * stage_bytes<BF16>();
@@ -629,12 +577,18 @@ cudaError_t launch(const Format &f, const float *X, int64_t ldx, int64_t batch, 
             break;
         }
     }
-    p.table = table;
-    p.nsets = nsets;
     const cudaError_t attr = allow_smem(xres_kernel<BF16, T>, kSmemCap);
     if (attr != cudaSuccess) return attr;
-    const int ncl = static_cast<int>(
-        std::min<int64_t>({int64_t(max_clusters<BF16, T>(p.C, smem)), int64_t(kMaxClusters), units}));
+    const int64_t occ = std::min<int64_t>(max_clusters<BF16, T>(p.C, smem), kMaxClusters);
+    // Row sets of about 4 heaviest groups (table 1: 128 rows and more, the
+    // consumers' efficient layout) when they still give every cluster 3 units or
+    // more; else sets of about 2 (table 0), whose finer units balance better.
+    const int table = tiles * f.nxsets[1] >= 3 * occ ? 1 : 0;
+    const int nsets = f.nxsets[table];
+    const int64_t units = tiles * nsets;
+    p.table = table;
+    p.nsets = nsets;
+    const int ncl = static_cast<int>(std::min<int64_t>(occ, units));
     if (ncl <= 0) return cudaErrorNotSupported;
     // contiguous runs of units of about equal time: cluster c starts at the
     // first unit whose cumulative cost reaches c / ncl of the total.  The ranks
