@@ -136,19 +136,13 @@ __device__ __forceinline__ void chunk(const unsigned char *s_vals, const uint32_
 #pragma unroll
                 for (int u = 0; u < KQ; ++u) {
                     const float4 xv = xr[u * LPR];
-                    acc[u].x = fmaf(v[e], xv.x, acc[u].x);
-                    acc[u].y = fmaf(v[e], xv.y, acc[u].y);
-                    acc[u].z = fmaf(v[e], xv.z, acc[u].z);
-                    acc[u].w = fmaf(v[e], xv.w, acc[u].w);
+                    fma4(acc[u], v[e], xv);
                 }
             } else {
 #pragma unroll
                 for (int u = 0; u < KQ; ++u) {
                     const float4 xv = xr[u * LPR];
-                    acc2[u].x = fmaf(v[e], xv.x, acc2[u].x);
-                    acc2[u].y = fmaf(v[e], xv.y, acc2[u].y);
-                    acc2[u].z = fmaf(v[e], xv.z, acc2[u].z);
-                    acc2[u].w = fmaf(v[e], xv.w, acc2[u].w);
+                    fma4(acc2[u], v[e], xv);
                 }
             }
         }
@@ -202,10 +196,7 @@ __device__ __forceinline__ void chunk_rows(const unsigned char *s_vals, const ui
 #pragma unroll
                 for (int u = 0; u < KQ; ++u) {
                     const float4 xv = xr[u * LPR];
-                    acc[p][u].x = fmaf(v, xv.x, acc[p][u].x);
-                    acc[p][u].y = fmaf(v, xv.y, acc[p][u].y);
-                    acc[p][u].z = fmaf(v, xv.z, acc[p][u].z);
-                    acc[p][u].w = fmaf(v, xv.w, acc[p][u].w);
+                    fma4(acc[p][u], v, xv);
                 }
             }
         }

@@ -16,6 +16,26 @@ namespace darb {
 
 constexpr int kWarps = 8;   // warps per CTA for the row-per-lane kernels
 
+// acc += v * x for a float4 accumulator with two packed fp32 FMAs (PTX
+// fma.rn.f32x2, sm_100 and later): each element is one IEEE fma, as fmaf,
+// in half the instructions.
+__device__ __forceinline__ void fma4(float4 &acc, float v, const float4 &x) {
+    asm("{\n"
+        " .reg .b64 vv, xl, xh, al, ah;\n"
+        " mov.b64 vv, {%8, %8};\n"
+        " mov.b64 xl, {%4, %5};\n"
+        " mov.b64 xh, {%6, %7};\n"
+        " mov.b64 al, {%0, %1};\n"
+        " mov.b64 ah, {%2, %3};\n"
+        " fma.rn.f32x2 al, vv, xl, al;\n"
+        " fma.rn.f32x2 ah, vv, xh, ah;\n"
+        " mov.b64 {%0, %1}, al;\n"
+        " mov.b64 {%2, %3}, ah;\n"
+        "}"
+        : "+f"(acc.x), "+f"(acc.y), "+f"(acc.z), "+f"(acc.w)
+        : "f"(x.x), "f"(x.y), "f"(x.z), "f"(x.w), "f"(v));
+}
+
 // The 8 kept values of (chunk c, slot i), widened to fp32 (bf16 -> fp32 is exact).
 template <bool BF16>
 __device__ __forceinline__ void load_chunk(const void *vals, int64_t idx, float (&v)[kChunk]) {

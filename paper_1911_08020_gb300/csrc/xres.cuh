@@ -425,20 +425,8 @@ xres_kernel(Format f, const float *__restrict__ X, int64_t batch, float *__restr
                                 else
                                     v = __uint_as_float(vw[e]);
                                 const uint32_t ad = xb + uint32_t(e) * mrow + (off << 7);
-                                const float4 xa = lds_f4(ad);
-                                float4 &a = accA[pp];
-                                a.x = fmaf(v, xa.x, a.x);
-                                a.y = fmaf(v, xa.y, a.y);
-                                a.z = fmaf(v, xa.z, a.z);
-                                a.w = fmaf(v, xa.w, a.w);
-                                if constexpr (kTwo) {
-                                    const float4 xc = lds_f4(ad ^ 64u);   // the other half of the row
-                                    float4 &b = accB[pp];
-                                    b.x = fmaf(v, xc.x, b.x);
-                                    b.y = fmaf(v, xc.y, b.y);
-                                    b.z = fmaf(v, xc.z, b.z);
-                                    b.w = fmaf(v, xc.w, b.w);
-                                }
+                                fma4(accA[pp], v, lds_f4(ad));
+                                if constexpr (kTwo) fma4(accB[pp], v, lds_f4(ad ^ 64u));   // the other half of the row
                             };
                             if (e_lo == 0 && e_hi == kChunk) {
                                 // a whole chunk: one straight run, every load can be issued early
