@@ -47,6 +47,12 @@ def parse_args():
     p.add_argument("--no-cpu", action="store_true")
     p.add_argument("--no-rnn", action="store_true")
     p.add_argument("--no-baselines", action="store_true", help="skip the cuSPARSE comparison section")
+    p.add_argument("--step-only", action="store_true",
+                   help="time the step and its calls only (no tensor-core, gemv_1024, RNN, assignment or "
+                        "baseline sections): the run whose launch list the profiles summarise")
+    p.add_argument("--path", choices=("auto", "tensor"), default="auto",
+                   help="kernel family of the products: darb_spmm (auto), or the opt-in tensor-core path "
+                        "(darb_spmm_ex with DARB_PATH_TENSOR_CORES; for profiling it)")
     p.add_argument("--calls", default="",
                    help="comma list restricting the step to some calls, e.g. fc6_spmm_b256 (profiling)")
     return p.parse_args()
@@ -372,8 +378,9 @@ def roofline(wl, di, dom, dom_ms, achieved, peak, peak_kind, tpeak, tpeak_kind, 
 class Workload:
     """Rotating sets of device buffers for the FC6/FC7 step."""
 
-    def __init__(self, torch, darb, synth, only=()):
+    def __init__(self, torch, darb, synth, only=(), path="auto"):
         self.torch, self.darb = torch, darb
+        self.tensor = path == "tensor"
         wl = synth.WORKLOADS[WORKLOAD]
         dev = torch.device("cuda", torch.cuda.current_device())
         self.dev = dev
@@ -415,6 +422,8 @@ class Workload:
         for kind, mi, b, _ in self.calls:
             if kind == "encode":
                 self.paths.append(("encode", 1))
+            elif self.tensor:
+                self.paths.append(("tensor", 2))   # split_kernel + tc_kernel
             else:
                 path, kernels = darb.darb_spmm_path(self.mats[mi]["h"], b)
                 self.paths.append(("tensor" if path == darb.PATH_TENSOR_CORES else "cuda", kernels))
@@ -425,6 +434,9 @@ class Workload:
         st = self.sets[s % NSETS]
         if kind == "encode":
             self.darb.darb_reencode(st["enc"][mi], st["W"][mi], stream)
+        elif self.tensor:
+            self.darb.darb_spmm_ex(st["spmm"][(mi, b)], st["X"][(mi, b)], st["Y"][(mi, b)],
+                                   self.darb.PATH_TENSOR_CORES, stream)
         else:
             self.darb.darb_spmm(st["spmm"][(mi, b)], st["X"][(mi, b)], st["Y"][(mi, b)], stream)
 
@@ -451,7 +463,7 @@ def run_gpu(args, world, rank, local):
     from paper_1911_08020_gb300 import darb, synth
     torch.cuda.set_device(local)
     only = tuple(c for c in args.calls.split(",") if c)
-    wl = Workload(torch, darb, synth, only)
+    wl = Workload(torch, darb, synth, only, args.path)
     stream = torch.cuda.current_stream()
     sid = stream.cuda_stream
     ncalls = len(wl.calls)
@@ -584,13 +596,14 @@ def run_gpu(args, world, rank, local):
         "gpu_launches": wl.step_launches * args.steps,
         "clocks": clocks,
     }
-    if not only:
+    extras = not only and not args.step_only
+    if extras:
         result["tensor_cores"] = run_tensor(torch, darb, wl, stream)
         result["gemv_1024"] = run_gemv_1024(torch, darb, synth, peak, stream)
-    if not args.no_rnn and not only:
+    if not args.no_rnn and extras:
         result["rnn"] = run_rnn(torch, darb, synth, peak)
         result["assign"] = run_assign(torch, darb, wl, peak)
-    if not args.no_baselines and not only:
+    if not args.no_baselines and extras:
         result["baselines"] = run_baselines(torch, darb, wl)
     if not args.no_e2e:
         result["e2e"] = run_e2e(args, wl, torch, darb)
