@@ -490,11 +490,20 @@ batch_kernel(Format f, const WorkItem *__restrict__ items, const float *__restri
     for (int idx = tid; idx < (s1 - s0) * kBt * kParts; idx += kThreads) {
         const int s = s0 + idx / (kBt * kParts), pt = (idx / kBt) % kParts, t = idx % kBt;
         const int gi = s / kSlots, slot = s % kSlots;
+        // every rank's partial sum requested before any is added (one round trip
+        // through distributed shared memory, not one per rank), with the row's
+        // map entry and its group's row count alongside
+        const int pidx = (s * kParts + pt) * kBt + t;
+        float pv[8];
+#pragma unroll
+        for (int r = 0; r < 8; ++r)
+            if (r < ksub) pv[r] = (ksc > 1 ? cluster.map_shared_rank(part, qbase + r) : part)[pidx];
+        const int row = f.rowmap[(gfirst + gi) * kSlots + slot];
         if (b0 + t >= batch || slot >= f.groups[gfirst + gi].nrows) continue;
         float sum = 0.0f;   // ranks in a fixed order: deterministic
-        for (int r = 0; r < ksub; ++r)
-            sum += (ksc > 1 ? cluster.map_shared_rank(part, qbase + r) : part)[(s * kParts + pt) * kBt + t];
-        const int row = f.rowmap[(gfirst + gi) * kSlots + slot];
+#pragma unroll
+        for (int r = 0; r < 8; ++r)
+            if (r < ksub) sum += pv[r];
         if constexpr (MODE == kModeY) Y[int64_t(row) * ldy + b0 + t] = sum;
         else (pt == 0 ? ra.gx : ra.gh)[int64_t(row) * ra.B + b0 + t] = sum;
     }

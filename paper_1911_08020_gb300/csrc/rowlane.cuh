@@ -231,9 +231,17 @@ rowlane_kernel(Format f, const float *__restrict__ X, int64_t ldx, int64_t batch
     const int s0 = min(g.nrows, q * per), s1 = min(g.nrows, s0 + per);
     for (int idx = tid; idx < (s1 - s0) * kPb; idx += kWarps * 32) {
         const int slot = s0 + idx / kPb, t = idx % kPb;
-        float s = 0.0f;
-        for (int r = 0; r < ksc; ++r) s += (ksc > 1 ? cluster.map_shared_rank(s_part, r) : s_part)[slot * kPb + t];
+        // every rank's partial sum requested before any is added: one round trip
+        // through distributed shared memory, not one per rank
+        float pv[8];
+#pragma unroll
+        for (int r = 0; r < 8; ++r)
+            if (r < ksc) pv[r] = (ksc > 1 ? cluster.map_shared_rank(s_part, r) : s_part)[slot * kPb + t];
         const int row = f.rowmap[gi * kSlots + slot];
+        float s = 0.0f;
+#pragma unroll
+        for (int r = 0; r < 8; ++r)
+            if (r < ksc) s += pv[r];
         if constexpr (MODE == kModeY) {
             if (t < nb) Y[int64_t(row) * ldy + t] = s;
         } else {
