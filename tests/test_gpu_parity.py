@@ -109,6 +109,39 @@ def test_encode_strided_and_misaligned_rows():
                 darb.darb_destroy(h)
 
 
+@pytest.mark.parametrize("mset", [(8,), (128, 256), (8, 16, 32, 64, 128, 256)])
+def test_encode_bf16_power_of_two_block_sizes(mset):
+    """bf16 weights whose block sizes are all powers of two from 8 to 256, in
+    rows padded to a multiple of 8 elements: the encoder's row path (tiles of
+    2048 columns, one 16-byte unit per lane; several lanes per block above
+    m = 64).  Every row length, so that a row's last block and last 8-element
+    unit may be partial; Gaussian, tied, signed-zero and infinite weights; the
+    padding past each row holds NaNs, which must never be read."""
+    g = np.random.default_rng(14)
+    for rows, cols in ((1, 8), (3, 17), (33, 100), (64, 1000), (40, 2049), (7, 4296), (5, 12289)):
+        ldw = (cols + 7) // 8 * 8 + 8
+        for mode in range(4):
+            if mode == 1:
+                w = np.round(g.standard_normal((rows, cols)) * 2).astype(np.float32)       # many ties
+            elif mode == 2:
+                w = np.where(g.random((rows, cols)) < 0.5, 0.0, -0.0).astype(np.float32)  # all +-0
+            else:
+                w = g.standard_normal((rows, cols)).astype(np.float32)
+                if mode == 3:
+                    w[g.random((rows, cols)) < 0.05] = np.inf
+                    w[g.random((rows, cols)) < 0.05] = -np.inf
+            m = g.choice(np.asarray(mset, np.int32), size=rows)
+            stored = synth.f32_to_bf16_bits(w)
+            big = np.full((rows, ldw), 0x7FC1, np.uint16)   # NaN past each row's end
+            big[:, :cols] = stored
+            Wt = weight_tensor(big, "bf16")[:, :cols]
+            h = darb.darb_encode(Wt, m)
+            try:
+                assert_encoding_equal(h, oracle.encode(stored, m, "bf16"))
+            finally:
+                darb.darb_destroy(h)
+
+
 def test_encode_nan_is_reported():
     w = np.ones((40, 64), np.float32)
     w[37, 61] = np.nan
