@@ -164,6 +164,12 @@ cudaError_t launch_spmm_tc(const Format &f, const float *X, int64_t ldx, int64_t
 // `path`: a darb_path_t; DARB_PATH_AUTO and DARB_PATH_CUDA_CORES both take the
 // CUDA-core gather.  cudaErrorNotSupported if DARB_PATH_TENSOR_CORES was asked
 // for a call the tensor-core kernel cannot take.
+// Y = (the first col_limit columns of W_darb) (the first col_limit rows of X),
+// for X whose rows from col_limit on are zero: the product of launch_spmm,
+// on xres without the columns from col_limit on where it can take the call.
+cudaError_t launch_spmm_prefix(const Format &f, int64_t col_limit, const float *X, int64_t ldx, int64_t batch,
+                               float *Y, int64_t ldy, bool early, cudaStream_t stream);
+
 cudaError_t launch_spmm(const Format &f, const float *X, int64_t ldx, int64_t batch, float *Y,
                         int64_t ldy, bool early, int path, cudaStream_t stream);
 

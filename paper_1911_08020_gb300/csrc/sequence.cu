@@ -740,7 +740,8 @@ static cudaError_t launch_seq_t(const Format &f, const int32_t *row_m, seq::SeqA
             gather_x_kernel<<<grid, 256, 0, stream>>>(a.x, a.T, I, B, xall, ldx);
             e = cudaGetLastError();
         }
-        if (e == cudaSuccess) e = launch_spmm(f, xall, ldx, T * B, gx, ldx, false, DARB_PATH_AUTO, stream);
+        // only the x columns: xall's h rows are zero
+        if (e == cudaSuccess) e = launch_spmm_prefix(f, I, xall, ldx, T * B, gx, ldx, false, stream);
         a.gx = gx;
         a.ldgx = ldx;
     }

@@ -546,7 +546,9 @@ cudaError_t launch(const Format &f, const float *X, int64_t ldx, int64_t batch, 
     for (int C = 1;; C *= 2) {
         if (C > 8) return cudaErrorNotSupported;
         const int64_t S = (f.cols + C - 1) / C;
-        const int64_t rows = std::min<int64_t>(f.cols, S + f.m_max - 1);
+        // a slice's blocks start in [q S, (q + 1) S) and select rows up to m_max - 1
+        // further (rows past the matrix arrive as zeros)
+        const int64_t rows = S + f.m_max - 1;
         const int nboxes = static_cast<int>((rows + 255) / 256);
         int box_rows = static_cast<int>((rows + nboxes - 1) / nboxes);
         const uint64_t x_bytes = uint64_t(nboxes) * box_rows * T * 4;
