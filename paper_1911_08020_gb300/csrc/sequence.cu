@@ -69,6 +69,12 @@ struct SeqArgs {
     float *c_seq;           // T x H x B or nullptr (LSTM)
     float *c_state;         // H x B: the running cell state when it is not on chip (LSTM)
     float *c_last;          // H x B or nullptr (LSTM)
+    // a copy of h_t with rows of ldp columns (B rounded up to the batch tile,
+    // zeros past B) in two buffers by step parity, H x ldp each, or nullptr:
+    // h_{t-1} is then staged from h_seq.  Boxes over it are whole 128-byte
+    // aligned rows; boxes over B-column rows with a ragged tail are not
+    float *h_pad;
+    int64_t ldp;
     unsigned *bar;          // arrival counter, zero at launch
     int *abort_flag;        // zero at launch
     int32_t *status;
@@ -429,7 +435,7 @@ seq_kernel(Format f, SeqArgs a, Ranges rg, SmemPlan sp, const __grid_constant__ 
                     const int y = isx ? bx * a.bxh : (bx - a.nbx) * a.bhh;
                     float *dst = s_in + (int64_t(isx ? y : a.ipad + y) << lbt);
                     const CUtensorMap *m = isx ? &mx : (t == 0 ? &mh0 : &mhs);
-                    const int z = isx ? t : (t == 0 ? 0 : t - 1);
+                    const int z = isx ? t : (t == 0 ? 0 : (a.h_pad ? (t - 1) & 1 : t - 1));
                     tensor3d_g2s(dst, m, static_cast<int>(b0), y, z, &s_full);
                 }
                 bool ok = mbar_wait(&s_full, tile & 1, false);
@@ -484,7 +490,11 @@ seq_kernel(Format f, SeqArgs a, Ranges rg, SmemPlan sp, const __grid_constant__ 
             };
             for (int i = tid; i < nu << lbt; i += kThreads) {
                 const int ui = i >> lbt, j = i & (bt - 1);
-                if (j >= nb) continue;
+                float *hq = a.h_pad ? a.h_pad + (int64_t(t & 1) * H + u0 + ui) * a.ldp + b0 + j : nullptr;
+                if (j >= nb) {
+                    if (hq) *hq = 0.0f;
+                    continue;
+                }
                 const int64_t e = int64_t(ui) * B + b0 + j;
                 auto xg = [&](int lr) { return pre ? s_gx[(lr << lbt) + j] : 0.0f; };
                 if constexpr (MODE == kModeLstm) {
@@ -493,7 +503,9 @@ seq_kernel(Format f, SeqArgs a, Ranges rg, SmemPlan sp, const __grid_constant__ 
                     const float c = sigm(pf) * cp[e] + sigm(pi) * tanhf(pg);
                     c_run[e] = c;
                     if (ct) ct[e] = c;
-                    ht[e] = sigm(po) * tanhf(c);
+                    const float hv = sigm(po) * tanhf(c);
+                    ht[e] = hv;
+                    if (hq) *hq = hv;
                 } else {
                     // x part (b_ih + W_x x) and h part (b_hh + W_h h) of each gate
                     auto gx_ = [&](int lr) { return s_bias[lr] + (pre ? xg(lr) : sum(lr, 0, j)); };
@@ -501,7 +513,9 @@ seq_kernel(Format f, SeqArgs a, Ranges rg, SmemPlan sp, const __grid_constant__ 
                     const float rr = sigm(gx_(ui) + gh_(ui));
                     const float zz = sigm(gx_(nu + ui) + gh_(nu + ui));
                     const float nn = tanhf(gx_(2 * nu + ui) + rr * gh_(2 * nu + ui));
-                    ht[e] = (1.0f - zz) * nn + zz * s_in[((a.ipad + u0 + ui) << lbt) + j];
+                    const float hv = (1.0f - zz) * nn + zz * s_in[((a.ipad + u0 + ui) << lbt) + j];
+                    ht[e] = hv;
+                    if (hq) *hq = hv;
                 }
             }
             __syncthreads();
@@ -682,28 +696,6 @@ static cudaError_t launch_seq_t(const Format &f, const int32_t *row_m, seq::SeqA
     else if (ptrs && B == 1 && xrows % 4 == 0 && H % 4 == 0) a.stage_mode = kStageQuadRows;
     const cudaError_t attr = allow_smem(seq_kernel<BF16, MODE>, kSmemCap);
     if (attr != cudaSuccess) return attr;
-    // tensor maps of the staged sources: 3-D (batch, rows, step) so that a box
-    // running past the last row of a step reads zeros, never the next step
-    CUtensorMap mx{}, mh0{}, mhs{};
-    if (a.tma) {
-        auto make = [&](CUtensorMap *m, const float *base, int64_t rows, int64_t depth, int boxh) {
-            const cuuint64_t dims[3] = {cuuint64_t(B), cuuint64_t(rows), cuuint64_t(depth)};
-            const cuuint64_t strides[2] = {cuuint64_t(B) * 4, cuuint64_t(B) * 4 * cuuint64_t(rows)};
-            const cuuint32_t box[3] = {cuuint32_t(bt), cuuint32_t(boxh), 1};
-            const cuuint32_t es[3] = {1, 1, 1};
-            return tensor_map_encoder()(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3, const_cast<float *>(base), dims,
-                                        strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
-                                        CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-                                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
-        };
-        bool ok = make(&mh0, a.h0, H, 1, bhh) && make(&mhs, a.h_seq, H, T, bhh);
-        if (ok && nbx) ok = make(&mx, a.x, I, T, bxh);
-        if (!ok) {   // plain loads instead (the plan above has room for either)
-            a.tma = 0;
-            a.ipad = xrows;
-            a.hpad = H;
-        }
-    }
     cudaLaunchAttribute at[1];
     at[0].id = cudaLaunchAttributeCooperative;
     at[0].val.cooperative = 1;
@@ -720,9 +712,12 @@ static cudaError_t launch_seq_t(const Format &f, const int32_t *row_m, seq::SeqA
     a.skip_cta = -1;
     sequence_test_hook(&a.barrier_ns, &a.skip_cta);
     // workspace: barrier word and abort flag; the cell state when it is neither
-    // on chip nor in c_last; the x parts and the product input they come from
+    // on chip nor in c_last; the x parts and the product input they come from;
+    // the padded copy of h_t
     const size_t cbytes = kGru || c_on_chip || c_last ? 0 : up(size_t(H) * size_t(B) * 4);
-    const size_t ws_bytes = 256 + cbytes + (pre ? pre_bytes : 0);
+    const int64_t ldp = (B + bt - 1) / bt * bt;
+    const size_t pbytes = a.tma && ldp != B && T > 1 ? up(2 * size_t(H) * size_t(ldp) * 4) : 0;
+    const size_t ws_bytes = 256 + cbytes + (pre ? pre_bytes : 0) + pbytes;
     char *ws = nullptr;
     cudaError_t e = stream_alloc(reinterpret_cast<void **>(&ws), ws_bytes, stream);
     if (e != cudaSuccess) return e;
@@ -730,6 +725,8 @@ static cudaError_t launch_seq_t(const Format &f, const int32_t *row_m, seq::SeqA
     a.bar = reinterpret_cast<unsigned *>(ws);
     a.abort_flag = reinterpret_cast<int *>(ws + 4);
     a.c_state = kGru || c_on_chip ? nullptr : (c_last ? c_last : reinterpret_cast<float *>(ws + 256));
+    a.h_pad = pbytes ? reinterpret_cast<float *>(ws + ws_bytes - pbytes) : nullptr;
+    a.ldp = ldp;
     if (pre && e == cudaSuccess) {
         float *xall = reinterpret_cast<float *>(ws + 256 + cbytes);
         float *gx = reinterpret_cast<float *>(ws + 256 + cbytes + up(size_t(I + H) * ldx * 4));
@@ -744,6 +741,31 @@ static cudaError_t launch_seq_t(const Format &f, const int32_t *row_m, seq::SeqA
         if (e == cudaSuccess) e = launch_spmm_prefix(f, I, xall, ldx, T * B, gx, ldx, false, stream);
         a.gx = gx;
         a.ldgx = ldx;
+    }
+    // tensor maps of the staged sources: 3-D (batch, rows, step) so that a box
+    // running past the last row of a step reads zeros, never the next step;
+    // h_{t-1} from the padded copy when the last batch tile is ragged
+    CUtensorMap mx{}, mh0{}, mhs{};
+    if (a.tma && e == cudaSuccess) {
+        auto make = [&](CUtensorMap *m, const float *base, int64_t cols, int64_t rows, int64_t depth, int boxh) {
+            const cuuint64_t dims[3] = {cuuint64_t(cols), cuuint64_t(rows), cuuint64_t(depth)};
+            const cuuint64_t strides[2] = {cuuint64_t(cols) * 4, cuuint64_t(cols) * 4 * cuuint64_t(rows)};
+            const cuuint32_t box[3] = {cuuint32_t(bt), cuuint32_t(boxh), 1};
+            const cuuint32_t es[3] = {1, 1, 1};
+            return tensor_map_encoder()(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3, const_cast<float *>(base), dims,
+                                        strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+                                        CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+        };
+        bool ok = make(&mh0, a.h0, B, H, 1, bhh) &&
+                  (a.h_pad ? make(&mhs, a.h_pad, a.ldp, H, 2, bhh) : make(&mhs, a.h_seq, B, H, T, bhh));
+        if (ok && nbx) ok = make(&mx, a.x, B, I, T, bxh);
+        if (!ok) {   // plain loads instead (the plan above has room for either)
+            a.tma = 0;
+            a.ipad = xrows;
+            a.hpad = H;
+            a.h_pad = nullptr;
+        }
     }
     if (e == cudaSuccess) e = cudaLaunchKernelEx(&cfg, seq_kernel<BF16, MODE>, f, a, rg, sp, mx, mh0, mhs);
     const cudaError_t ef = cudaFreeAsync(ws, stream);

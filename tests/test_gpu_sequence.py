@@ -71,7 +71,8 @@ def _check_gru_sequence(h, ref, T, I, H, B, xs, h0, bi, bh, tol):
 
 # (I, H, B): one unit per CTA, ragged batch tiles, several tiles, I = 0, more
 # units than CTAs, a batch tile of one column; batches that are multiples of 4
-# stage through tensor maps (one CTA, clusters of two, a ragged second tile)
+# stage through tensor maps (one CTA; a ragged last tile staged from the padded
+# copy of h, as one tile (B = 12) and as the second of two (B = 40))
 SHAPES = [(0, 5, 1), (3, 4, 2), (7, 33, 3), (20, 40, 8), (64, 100, 9), (10, 70, 33), (16, 300, 1),
           (40, 200, 70), (5, 400, 17), (4, 1, 8), (6, 9, 4), (12, 36, 40), (0, 64, 12), (300, 260, 4)]
 
