@@ -252,7 +252,7 @@ void build_work_tables(darb_handle_s *h) {
         for (const int2 &s : sets) h->set_prefix[l].push_back(h->set_prefix[l].back() + s.y * nch_of(s));
     }
     // Row sets of xres: each bin's groups in runs of G = the largest power of
-    // two <= 8 with G * nch(bin) <= base * nch(heaviest bin), so that every set
+    // two <= kXresMaxGroups with G * nch(bin) <= base * nch(heaviest bin), so that every set
     // is about `base` groups of the heaviest bin's work; bins in layout order
     // (heaviest first).
     h->xsets.clear();
@@ -268,7 +268,7 @@ void build_work_tables(darb_handle_s *h) {
             const Group &g = h->groups[gbeg];
             const int64_t nch = ceil_div(g.n, kChunk);
             int G = 1;
-            while (2 * G <= 8 && 2 * G * nch <= base * nch_max) G *= 2;
+            while (2 * G <= darb::kXresMaxGroups && 2 * G * nch <= base * nch_max) G *= 2;
             for (size_t s = gbeg; s < gend; s += static_cast<size_t>(G)) {
                 darb::SetGeo sg{};
                 const size_t ng = std::min<size_t>(static_cast<size_t>(G), gend - s);

@@ -61,15 +61,15 @@ struct WorkItem {
 };
 constexpr int kWorkLevels = 4;   // row sets of up to 1, 2, 4, 8 groups
 
-// A row set of the resident-activation product (xres.cuh): a run of ng <= 8
-// consecutive groups of one bin, in one 48-byte record (no dependent lookups).
+// A row set of the resident-activation product (xres.cuh): a run of
+// ng <= kXresMaxGroups consecutive groups of one bin, in one 48-byte record (no dependent lookups).
 // The groups of a bin have equal block counts, so group g0 + i starts i group
 // strides after the first: values at val_off + i * nch * 256, offsets at
 // off_off + i * nch * 32 * (nib ? 1 : 2) (nch = ceil(n / 8)); all groups are
 // full except possibly the last.
 struct __align__(16) SetGeo {
     int32_t g0;           // first group
-    int32_t ng;           // groups (1..8)
+    int32_t ng;           // groups (1..kXresMaxGroups)
     int32_t m, n;         // block size and blocks per row
     int32_t nib;          // 1: 4-bit offsets
     int32_t nrows_last;   // rows in use of the last group
@@ -78,6 +78,10 @@ struct __align__(16) SetGeo {
     int64_t pad;
 };
 constexpr int kXresTables = 2;   // row-set tables of xres: 2 and 4 groups of the heaviest bin
+// Groups of an xres row set, at most: its partial sums (128 rows x 32 columns)
+// are one 16 KB buffer, which leaves the activation slice room enough for
+// clusters of 6 on the widest layers
+constexpr int kXresMaxGroups = 4;
 constexpr int kWorkSplits = 4;   // clusters of 1, 2, 4, 8 CTAs
 
 // Everything a kernel needs to read an encoded matrix.
@@ -101,7 +105,7 @@ struct Format {
     // chunks per row) of sets [0, s); nitems[l][0] + 1 entries
     const int64_t *set_prefix[kWorkLevels];
     // row sets of xres (SetGeo): table i sizes the sets of every bin to about
-    // the work of 2 << i groups of the heaviest bin (at most 8 groups); device
+    // the work of 2 << i groups of the heaviest bin (at most kXresMaxGroups); device
     // records, and on the HOST the prefix sums of their work (group-chunks)
     const SetGeo *xsets[kXresTables];
     int32_t nxsets[kXresTables];

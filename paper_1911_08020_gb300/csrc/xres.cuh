@@ -7,14 +7,17 @@
 // columns of W into C slices of S columns; a block belongs to the slice its
 // first column falls in, so a CTA that holds rows [q*S, (q+1)*S + m_max - 1)
 // of the tile can multiply every block of its slice, of every row, without
-// staging anything else.  A cluster of C CTAs (one per slice) therefore loads
-// the tile once and then streams only the kept values and packed offsets
-// (2.5 bytes per kept weight for bf16) through a ring of bulk copies.  The C
-// partial sums of a row meet in distributed shared memory.
+// staging anything else (rows [q*S, (q+1)*S) when S is a multiple of every
+// block size: no block then reaches past its slice).  C is the split whose
+// clusters occupy the most SMs: clusters of 8 fill 120 of the 152, of 6 138,
+// of 4 144.  A cluster of C CTAs (one per slice) therefore loads the tile
+// once and then streams only the kept values and packed offsets (2.5 bytes
+// per kept weight for bf16) through a ring of bulk copies.  The C partial
+// sums of a row meet in distributed shared memory.
 //
 // Layout of the work:
 //  * persistent clusters (as many as the GPU holds at once), one CTA per SM;
-//  * a unit = (batch tile of T columns, row set): a run of up to 8 groups of
+//  * a unit = (batch tile of T columns, row set): a run of up to 4 groups of
 //    one block-size bin, sized so that every set has about the work of a
 //    fixed number of groups of the heaviest bin (the SetGeo tables of the
 //    handle); units in tile-major order; each cluster takes a contiguous run
@@ -23,16 +26,18 @@
 //    columns (two 16-byte loads per kept weight, so that one offset, one value
 //    and one address serve 8 FMAs; the two rows of a quarter-warp read
 //    opposite halves of their activation rows, which keeps the loads free of
-//    bank conflicts); a pass covers 128 rows, a thread owns 1 or 2 rows of the
-//    set;
+//    bank conflicts); a pass covers 128 rows, the largest set, and a thread
+//    owns one row of it;
 //  * one producer warp: bulk copies of the values and offsets of each round
-//    (a run of chunks of the set's groups) into a 6-stage ring with full /
-//    empty mbarriers, and tensor-map copies of the tile slice (rows past the
-//    matrix or columns past the batch arrive as zeros);
+//    (a run of chunks of the set's groups) into a ring of 3 to 6 stages (as
+//    many as fit beside the slice) with full / empty mbarriers, and
+//    tensor-map copies of the tile slice (rows past the matrix or columns
+//    past the batch arrive as zeros);
 //  * three reducer warps: when every CTA of the cluster has stored its partial
 //    sums of a set (each consumer warp, once its rows are stored, arrives on
-//    every CTA's "ready" barrier), they add, for this CTA's R/C rows, the C
-//    partial sums in rank order (deterministic), write Y, and each reducer
+//    every CTA's "ready" barrier), they add, for this CTA's share of the
+//    set's R rows ([q R / C, (q + 1) R / C)), the C partial sums in rank
+//    order (deterministic), write Y, and each reducer
 //    warp arrives on every CTA's "freed" barrier; the consumers meanwhile
 //    multiply the next set, and store its partial sums only once every CTA's
 //    reducers have read the previous ones.  No CTA-wide barrier separates
@@ -83,12 +88,13 @@ constexpr int kRWarps = 3;                     // reducer warps (20 warps in all
 constexpr int kRThreads = kRWarps * 32;
 constexpr int kProducerWarp = kCWarps;
 constexpr int kThreads = kCThreads + 32 + kRThreads;
-constexpr int kStages = 6;                     // rounds of values and offsets in the ring
+constexpr int kMaxStages = 6;                  // rounds of values and offsets in the ring, at most
+constexpr int kMinStages = 3;                  // and at least, unless nothing else fits
 constexpr int kRecCap = 8;                     // (group, chunk) records per round
-constexpr int kMaxGroups = 8;                  // groups of a row set, at most
+constexpr int kMaxGroups = kXresMaxGroups;     // groups of a row set, at most
 constexpr int kMaxClusters = 160;
 constexpr int kUnitCost = 10;                  // fixed cost of a unit, in group-chunks
-constexpr size_t kSmemCap = 226 * 1024;        // dynamic shared memory, at most
+constexpr size_t kSmemCap = 227 * 1024;        // dynamic shared memory, at most (the kernel has no static part)
 
 template <bool BF16>
 __host__ __device__ constexpr uint32_t rec_val_bytes() { return kSlots * kChunk * (BF16 ? 2 : 4); }
@@ -99,8 +105,9 @@ template <bool BF16>
 __host__ __device__ constexpr uint32_t stage_bytes() { return ring_val_bytes<BF16>() + kRecCap * kRecOffBytes; }
 
 struct Plan {
-    int C;            // CTAs per cluster = column slices
+    int C;            // CTAs per cluster = column slices (1 .. 8)
     int S;            // a slice's blocks start in columns [q*S, (q+1)*S)
+    int nst;          // stages of the ring (kMinStages or fewer only when nothing else fits)
     int box_rows;     // activation rows per tensor-map box
     int nboxes;       // boxes per slice
     int table;        // row-set table (SetGeo) of the handle
@@ -112,7 +119,7 @@ struct Plan {
 
 // Barriers at the start of dynamic shared memory.
 struct Bars {
-    uint64_t full[kStages], empty[kStages];
+    uint64_t full[kMaxStages], empty[kMaxStages];
     uint64_t xfull, xfree;
     uint64_t ready, freed;
 };
@@ -134,11 +141,11 @@ xres_kernel(Format f, const float *__restrict__ X, int64_t batch, float *__restr
     Bars &bar = *reinterpret_cast<Bars *>(sm);
     float *s_x = reinterpret_cast<float *>(sm + 128);
     unsigned char *s_ring = sm + p.ring_off;
-    float *s_part = reinterpret_cast<float *>(sm + p.part_off);   // [8 * 32 rows][T]
+    float *s_part = reinterpret_cast<float *>(sm + p.part_off);   // [kMaxGroups * 32 rows][T]
 
     pdl_launch_dependents();
     cg::cluster_group cluster = cg::this_cluster();
-    const int C = p.C;
+    const int C = p.C, NS = p.nst;
     const int q = static_cast<int>(cluster.block_rank());
     const int cl = static_cast<int>(blockIdx.x) / C;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -147,7 +154,7 @@ xres_kernel(Format f, const float *__restrict__ X, int64_t batch, float *__restr
     const int kq0 = q * p.S;                // first activation row of the slice
 
     if (tid == 0) {
-        for (int st = 0; st < kStages; ++st) {
+        for (int st = 0; st < NS; ++st) {
             mbar_init(&bar.full[st], 1);
             mbar_init(&bar.empty[st], kCWarps);
         }
@@ -227,6 +234,8 @@ xres_kernel(Format f, const float *__restrict__ X, int64_t batch, float *__restr
         // ------------------------------------------------------------ producer
         bool ok = true;
         int rc = 0;           // rounds issued
+        int pst = 0;          // the stage of round rc (rc % NS)
+        uint32_t pph = 0u;    // and the parity of its use ((rc / NS) & 1)
         int xloads = 0;       // slices loaded
         int cur_tile = -1;
         Cursor cu = cursor_at(u_begin), cn = cu;
@@ -254,8 +263,8 @@ xres_kernel(Format f, const float *__restrict__ X, int64_t batch, float *__restr
             const int rw = s.nib ? 1 : 2;
             const int64_t gnch = (s.n + kChunk - 1) / kChunk;   // chunks of a group
             for (int r = 0; r < g.rounds; ++r, ++rc) {
-                const int st = rc % kStages;
-                if (rc >= kStages) ok = mbar_wait(&bar.empty[st], ((rc / kStages) - 1) & 1, false);
+                const int st = pst;
+                if (rc >= NS) ok = mbar_wait(&bar.empty[st], pph ^ 1u, false);
                 ok = __shfl_sync(0xFFFFFFFFu, ok ? 1 : 0, 0) != 0;
                 if (!ok) break;
                 if (lane == 0) {
@@ -274,14 +283,18 @@ xres_kernel(Format f, const float *__restrict__ X, int64_t batch, float *__restr
                         bulk_g2s(so + size_t(gi) * bo, f.offs + oo, bo, &bar.full[st]);
                     }
                 }
+                if (++pst == NS) {
+                    pst = 0;
+                    pph ^= 1u;
+                }
             }
         }
         if (!ok && lane == 0) atomicOr(f.status, kStatusTimeout);
         // the copies this CTA started have landed before it can leave
         if (lane == 0) {
-            for (int k = 1; k <= kStages && k <= rc; ++k) {
+            for (int k = 1; k <= NS && k <= rc; ++k) {
                 const int last = rc - k;
-                mbar_wait(&bar.full[last % kStages], (last / kStages) & 1);
+                mbar_wait(&bar.full[last % NS], (last / NS) & 1);
             }
             if (xloads > 0) mbar_wait(&bar.xfull, (xloads - 1) & 1);
         }
@@ -298,9 +311,10 @@ xres_kernel(Format f, const float *__restrict__ X, int64_t batch, float *__restr
             if (ok) ok = mbar_wait_acq_cluster(&bar.ready, t & 1);
             if (ok) {
                 const int64_t tile = cu.tile;
-                const int rows_per = s.ng * kSlots / C;   // C divides 32
-                for (int i = rt; i < rows_per * (T / 4); i += kRThreads) {
-                    const int row = q * rows_per + i / (T / 4), c4 = i % (T / 4);
+                // this CTA's rows of the set: [q R / C, (q + 1) R / C)
+                const int R = s.ng * kSlots, r0 = q * R / C, r1 = (q + 1) * R / C;
+                for (int i = rt; i < (r1 - r0) * (T / 4); i += kRThreads) {
+                    const int row = r0 + i / (T / 4), c4 = i % (T / 4);
                     const int gg = row / kSlots, sl = row % kSlots;
                     if (gg == s.ng - 1 && sl >= s.nrows_last) continue;
                     const int idx = row * (T / 4) + c4;
@@ -352,6 +366,8 @@ xres_kernel(Format f, const float *__restrict__ X, int64_t batch, float *__restr
         //    one whole activation row.
         bool ok = true;
         int rc = 0, xloads = 0, cur_tile = -1;
+        int cst = 0;          // the stage of round rc (rc % NS)
+        uint32_t cph = 0u;    // and the parity of its use ((rc / NS) & 1)
         Cursor cu = cursor_at(u_begin), cn = cu;
         advance(cn);
         Set s_next = u_begin < u_end ? load_set(cu.sidx) : Set{};
@@ -385,8 +401,8 @@ xres_kernel(Format f, const float *__restrict__ X, int64_t batch, float *__restr
             }
             const uint32_t mrow = uint32_t(s.m) << 7;   // bytes between the first rows of consecutive blocks
             for (int r = 0; r < g.rounds; ++r, ++rc) {
-                const int st = rc % kStages;
-                if (ok) ok = mbar_wait(&bar.full[st], (rc / kStages) & 1, false);
+                const int st = cst;
+                if (ok) ok = mbar_wait(&bar.full[st], cph, false);
                 ok = __shfl_sync(0xFFFFFFFFu, ok ? 1 : 0, 0) != 0;
                 if (ok) {
                     const int cr0 = g.c0 + r * g.cpr, nchr = min(g.cpr, g.nch - r * g.cpr);
@@ -442,6 +458,10 @@ xres_kernel(Format f, const float *__restrict__ X, int64_t batch, float *__restr
                 }
                 __syncwarp();
                 if (lane == 0) mbar_arrive(&bar.empty[st]);
+                if (++cst == NS) {
+                    cst = 0;
+                    cph ^= 1u;
+                }
             }
             if (t >= 1 && ok) ok = mbar_wait_acq_cluster(&bar.freed, (t - 1) & 1);
 #pragma unroll
@@ -469,20 +489,16 @@ xres_kernel(Format f, const float *__restrict__ X, int64_t batch, float *__restr
             using L4 = std::integral_constant<int, 4>;
             using L8 = std::integral_constant<int, 8>;
             using N1 = std::integral_constant<int, 1>;
-            using N2 = std::integral_constant<int, 2>;
             using Nib = std::true_type;
             using Byte = std::false_type;
-            static_assert(2 * kCWarps * 8 >= kMaxGroups * kSlots, "two 128-row passes cover the largest set");
+            static_assert(kCWarps * 8 >= kMaxGroups * kSlots, "one 128-row pass covers the largest set");
             const int rows = s.ng * kSlots;
-            if (rows <= kCWarps * 4) {          // one pass of 8 lanes a row
+            if (rows <= kCWarps * 4) {   // one pass of 8 lanes a row
                 if (s.nib) unit(L8{}, N1{}, Nib{}, s, g, t);
                 else unit(L8{}, N1{}, Byte{}, s, g, t);
-            } else if (rows <= kCWarps * 8) {   // one pass of 4 lanes a row
+            } else {                     // one pass of 4 lanes a row
                 if (s.nib) unit(L4{}, N1{}, Nib{}, s, g, t);
                 else unit(L4{}, N1{}, Byte{}, s, g, t);
-            } else {
-                if (s.nib) unit(L4{}, N2{}, Nib{}, s, g, t);
-                else unit(L4{}, N2{}, Byte{}, s, g, t);
             }
             // this warp's partial sums are stored: tell every CTA's reducers
             __syncwarp();
@@ -527,7 +543,7 @@ inline int max_clusters(int C, uint32_t smem) {
 
 // The product on this kernel, or cudaErrorNotSupported when the call does not
 // fit it (the slice of the tile does not fit in shared memory even split 8
-// ways, or X cannot be described by a tensor map).
+// ways with a two-stage ring, or X cannot be described by a tensor map).
 template <bool BF16, int T>
 cudaError_t launch(const Format &f, const float *X, int64_t ldx, int64_t batch, float *Y, int64_t ldy, bool early,
                    cudaStream_t stream) {
@@ -539,36 +555,70 @@ cudaError_t launch(const Format &f, const float *X, int64_t ldx, int64_t batch, 
     if (reinterpret_cast<uintptr_t>(X) % 16 != 0 || (ldx * 4) % 16 != 0) return cudaErrorNotSupported;
     PFN_cuTensorMapEncodeTiled_v12000 enc = tensor_map_encoder();
     if (enc == nullptr) return cudaErrorNotSupported;
-    Plan p{};
-    uint32_t smem = 0;
-    // smallest split whose slice fits beside the ring and the partial sums of
-    // the largest set (8 groups)
-    for (int C = 1;; C *= 2) {
-        if (C > 8) return cudaErrorNotSupported;
-        const int64_t S = (f.cols + C - 1) / C;
-        // a slice's blocks start in [q S, (q + 1) S) and select rows up to m_max - 1
-        // further (rows past the matrix arrive as zeros)
-        const int64_t rows = S + f.m_max - 1;
-        const int nboxes = static_cast<int>((rows + 255) / 256);
-        int box_rows = static_cast<int>((rows + nboxes - 1) / nboxes);
-        const uint64_t x_bytes = uint64_t(nboxes) * box_rows * T * 4;
-        const uint64_t ring_off = 128 + x_bytes;
-        const uint64_t part_off = ring_off + uint64_t(kStages) * stage_bytes<BF16>();
-        const uint64_t total = part_off + uint64_t(kMaxGroups) * kSlots * T * 4;
-        if (total <= kSmemCap) {
-            p.C = C;
-            p.S = static_cast<int>(S);
-            p.box_rows = box_rows;
-            p.nboxes = nboxes;
-            p.x_bytes = static_cast<uint32_t>(x_bytes);
-            p.ring_off = static_cast<uint32_t>(ring_off);
-            p.part_off = static_cast<uint32_t>(part_off);
-            smem = static_cast<uint32_t>(total);
-            break;
-        }
-    }
     const cudaError_t attr = allow_smem(xres_kernel<BF16, T>, kSmemCap);
     if (attr != cudaSuccess) return attr;
+    // least common multiple of the block sizes (0 when it grows past any slice)
+    int64_t lcm = 1;
+    for (int i = 0; i < f.nxsets[0] && lcm != 0; ++i) {
+        const int64_t m = f.xsets_host[0][i].m;
+        int64_t a = lcm, b = m;
+        while (b != 0) {
+            const int64_t r = a % b;
+            a = b;
+            b = r;
+        }
+        lcm = lcm / a * m;
+        if (lcm > f.cols) lcm = 0;
+    }
+    // Per split C = 1 .. 8: slices of S columns.  A slice's blocks start in
+    // [q S, (q + 1) S) and select rows up to m_max - 1 past it (rows past the
+    // matrix arrive as zeros), unless S is a multiple of every block size: then
+    // no block crosses into the next slice and the slice is S rows, which is
+    // used whenever it is no longer.  Beside the slice: the deepest ring that
+    // fits (up to kMaxStages) and the partial sums of the largest set.  Of the
+    // splits with kMinStages or more, the one whose clusters occupy the most
+    // SMs, then the deeper ring, then the smaller split; a shallower ring only
+    // when no split has that.
+    Plan p{};
+    uint32_t smem = 0;
+    int64_t best_sms = 0;
+    int best_nst = 0;
+    bool best_deep = false;
+    for (int C = 1; C <= 8; ++C) {
+        int64_t S = (f.cols + C - 1) / C;
+        int64_t rows = S + f.m_max - 1;
+        if (lcm > 0) {
+            const int64_t Sa = (S + lcm - 1) / lcm * lcm;
+            if (Sa <= rows) S = rows = Sa;
+        }
+        const int nboxes = static_cast<int>((rows + 255) / 256);
+        const int box_rows = static_cast<int>((rows + nboxes - 1) / nboxes);
+        const uint64_t x_bytes = uint64_t(nboxes) * box_rows * T * 4;
+        const uint64_t ring_off = 128 + x_bytes;
+        const uint64_t part_bytes = uint64_t(kMaxGroups) * kSlots * T * 4;
+        if (ring_off + 2 * stage_bytes<BF16>() + part_bytes > kSmemCap) continue;
+        const int nst = static_cast<int>(
+            std::min<uint64_t>(kMaxStages, (kSmemCap - ring_off - part_bytes) / stage_bytes<BF16>()));
+        const uint64_t part_off = ring_off + uint64_t(nst) * stage_bytes<BF16>();
+        const uint32_t total = static_cast<uint32_t>(part_off + part_bytes);
+        const int64_t sms = std::min<int64_t>(max_clusters<BF16, T>(C, total), kMaxClusters) * C;
+        const bool deep = nst >= kMinStages;
+        const bool better = deep != best_deep ? deep : (sms != best_sms ? sms > best_sms : nst > best_nst);
+        if (sms <= 0 || !better) continue;
+        best_sms = sms;
+        best_nst = nst;
+        best_deep = deep;
+        p.C = C;
+        p.S = static_cast<int>(S);
+        p.nst = nst;
+        p.box_rows = box_rows;
+        p.nboxes = nboxes;
+        p.x_bytes = static_cast<uint32_t>(x_bytes);
+        p.ring_off = static_cast<uint32_t>(ring_off);
+        p.part_off = static_cast<uint32_t>(part_off);
+        smem = total;
+    }
+    if (best_sms <= 0) return cudaErrorNotSupported;
     const int64_t occ = std::min<int64_t>(max_clusters<BF16, T>(p.C, smem), kMaxClusters);
     // Row sets of about 4 heaviest groups (table 1: 128 rows and more, the
     // consumers' efficient layout) when they still give every cluster 3 units or

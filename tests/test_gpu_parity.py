@@ -207,6 +207,28 @@ def test_spmm_batches_and_ragged(dtype):
             darb.darb_destroy(h)
 
 
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_spmm_wide_column_slices(dtype):
+    """Wide matrices at batches above 16, where the columns are split over a
+    cluster: block sizes whose least common multiple divides the slice (no
+    block crosses a slice; the last slice runs past the matrix at 7000 and
+    9000 columns), one that divides it exactly (7000 columns, m in {10, 20,
+    40}), and sizes whose slices need the rows past their end (m up to 200)."""
+    g = np.random.default_rng(25)
+    for rows, cols, mset in ((300, 7000, (16, 32, 64)), (300, 7000, (10, 20, 40)), (260, 9000, (16, 64, 256)),
+                             (200, 6000, (3, 7, 16, 200)), (130, 12000, (8, 32))):
+        stored, m = _random_case(g, rows, cols, dtype, mset)
+        h, ref = encode_both(stored, m, dtype)
+        try:
+            for B in (17, 40, 64):
+                X = synth.activations(cols, B, seed=B + cols)
+                Y = darb.darb_spmm(h, t(X)).cpu().numpy()
+                Yr, A = oracle.darb_spmm(ref, X, with_absdot=True)
+                assert_product_close(Y, Yr, A, TOL[dtype])
+        finally:
+            darb.darb_destroy(h)
+
+
 def test_spmm_leading_dimensions_and_alignment():
     g = np.random.default_rng(21)
     rows, cols = 130, 300
