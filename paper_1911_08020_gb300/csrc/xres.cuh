@@ -94,6 +94,7 @@ constexpr int kRecCap = 8;                     // (group, chunk) records per rou
 constexpr int kMaxGroups = kXresMaxGroups;     // groups of a row set, at most
 constexpr int kMaxClusters = 160;
 constexpr int kUnitCost = 10;                  // fixed cost of a unit, in group-chunks
+constexpr int kSwitchCost = 40;                // a run's move to another batch tile, in group-chunks
 constexpr size_t kSmemCap = 227 * 1024;        // dynamic shared memory, at most (the kernel has no static part)
 
 template <bool BF16>
@@ -630,13 +631,17 @@ cudaError_t launch(const Format &f, const float *X, int64_t ldx, int64_t batch, 
     p.nsets = nsets;
     const int ncl = static_cast<int>(std::min<int64_t>(occ, units));
     if (ncl <= 0) return cudaErrorNotSupported;
-    // contiguous runs of units of about equal time: cluster c starts at the
-    // first unit whose cumulative cost reaches c / ncl of the total.  The ranks
-    // of a cluster go through a unit together, so a unit costs what its
-    // busiest rank streams -- its set's groups times the most chunks any
-    // slice's blocks touch -- plus a fixed cost per unit (the hand-off of its
-    // partial sums and the start of its rounds: about kUnitCost group-chunks
-    // of multiplying, measured on FC6/FC7).
+    // Contiguous runs of units, at most ncl of them, whose longest is as short
+    // as it can be.  The ranks of a cluster go through a unit together, so a
+    // unit costs what its busiest rank streams -- its set's groups times the
+    // most chunks any slice's blocks touch -- plus a fixed cost per unit (the
+    // hand-off of its partial sums and the start of its rounds); a run that
+    // crosses into the next batch tile also pays for the drain of its
+    // consumers and the load of the new slice.  kUnitCost and kSwitchCost
+    // were swept on FC6/FC7 at batch 64 and 256 (10 and 40 group-chunks of
+    // multiplying).  The bound on a run is found by bisection, each candidate
+    // tried by a greedy pass that closes a run where the next unit would pass
+    // it.
     thread_local std::vector<int64_t> cost;   // host; reused across calls
     const SetGeo *hs = f.xsets_host[table];
     cost.assign(static_cast<size_t>(nsets) + 1, 0);
@@ -651,17 +656,31 @@ cudaError_t launch(const Format &f, const float *X, int64_t ldx, int64_t batch, 
         cost[static_cast<size_t>(s) + 1] = cost[static_cast<size_t>(s)] + hs[s].ng * most + kUnitCost;
     }
     const int64_t *pre = cost.data();
-    const int64_t wt = pre[nsets];
-    const int64_t wtot = wt * tiles;
-    auto first_unit = [&](int c) -> int64_t {
-        if (c >= ncl) return units;
-        const int64_t target = (wtot * c + ncl - 1) / ncl;   // first unit with start >= target
-        const int64_t tile = target / wt, rem = target % wt;
-        const int64_t s = std::lower_bound(pre, pre + nsets, rem) - pre;
-        return tile * nsets + s;
+    auto unit_cost = [&](int64_t u) {
+        const int64_t sidx = u % nsets;
+        return pre[sidx + 1] - pre[sidx] + (sidx == 0 ? kSwitchCost : 0);
     };
-    for (int c = 0; c < ncl; ++c)
-        p.range[c] = make_int2(static_cast<int>(first_unit(c)), static_cast<int>(first_unit(c + 1)));
+    // (the switch is charged to a unit that opens a batch tile inside a run; a
+    // run's own first unit is charged its work alone)
+    auto greedy = [&](int64_t bound, bool write) {
+        int c = 0;
+        for (int64_t u = 0; u < units; ++c) {
+            const int64_t u0 = u;
+            int64_t acc = pre[u % nsets + 1] - pre[u % nsets];
+            for (++u; u < units && acc + unit_cost(u) <= bound; ++u) acc += unit_cost(u);
+            if (write) p.range[c] = make_int2(static_cast<int>(u0), static_cast<int>(u));
+        }
+        return c;
+    };
+    int64_t lo = 0, hi = 0;
+    for (int sidx = 0; sidx < nsets; ++sidx) lo = std::max<int64_t>(lo, pre[sidx + 1] - pre[sidx]);
+    for (int64_t u = 0; u < units; ++u) hi += unit_cost(u);
+    while (lo < hi) {   // the smallest bound whose runs fit ncl clusters
+        const int64_t mid = lo + (hi - lo) / 2;
+        if (greedy(mid, false) <= ncl) hi = mid;
+        else lo = mid + 1;
+    }
+    const int nrun = greedy(lo, true);
     CUtensorMap xmap;
     std::memset(&xmap, 0, sizeof xmap);
     const cuuint64_t dims[2] = {cuuint64_t(batch), cuuint64_t(f.cols)};
@@ -672,7 +691,7 @@ cudaError_t launch(const Format &f, const float *X, int64_t ldx, int64_t batch, 
             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
         return cudaErrorNotSupported;
-    return launch_ex(xres_kernel<BF16, T>, dim3(static_cast<unsigned>(ncl * p.C)), dim3(kThreads), smem, stream,
+    return launch_ex(xres_kernel<BF16, T>, dim3(static_cast<unsigned>(nrun * p.C)), dim3(kThreads), smem, stream,
                      static_cast<unsigned>(p.C), true, f, X, batch, Y, ldy, xmap, p);
 }
 
