@@ -32,7 +32,11 @@
 //    (a run of chunks of the set's groups) into a ring of 3 to 6 stages (as
 //    many as fit beside the slice) with full / empty mbarriers, and
 //    tensor-map copies of the tile slice (rows past the matrix or columns
-//    past the batch arrive as zeros);
+//    past the batch arrive as zeros), box by box, each box on its own
+//    barrier: a round waits only for the boxes holding the rows its blocks
+//    can select, so the consumers start on the first rows while the rest
+//    land; a run's first slice is requested before its first set record is
+//    read;
 //  * three reducer warps: when every CTA of the cluster has stored its partial
 //    sums of a set (each consumer warp, once its rows are stored, arrives on
 //    every CTA's "ready" barrier), they add, for this CTA's share of the
@@ -75,7 +79,7 @@ namespace cg = cooperative_groups;
 
 // 16 bytes of the staged activation slice at a 32-bit shared address.  Not
 // volatile: the address depends on offsets read after the stage's wait, and
-// the slice itself changes only across a wait on xfull.
+// the slice itself changes only across the waits on its boxes.
 __device__ __forceinline__ float4 lds_f4(uint32_t addr) {
     float4 v;
     asm("ld.shared.v4.f32 {%0, %1, %2, %3}, [%4];" : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w) : "r"(addr));
@@ -119,12 +123,15 @@ struct Plan {
 };
 
 // Barriers at the start of dynamic shared memory.
+constexpr int kMaxBoxes = 8;       // tensor-map boxes of a slice, at most (1816 rows of 128 bytes fill 227 KB)
+constexpr uint32_t kBarBytes = 256; // the barriers, in front of the slice
 struct Bars {
     uint64_t full[kMaxStages], empty[kMaxStages];
-    uint64_t xfull, xfree;
+    uint64_t xbox[kMaxBoxes];   // box i of the slice has landed
+    uint64_t xfree;             // the consumers are done with the slice
     uint64_t ready, freed;
 };
-static_assert(sizeof(Bars) <= 128, "the barriers fit in front of the slice");
+static_assert(sizeof(Bars) <= kBarBytes, "the barriers fit in front of the slice");
 
 // A row set as the kernel keeps it in registers (constant indexing only).
 struct Set {
@@ -140,7 +147,7 @@ xres_kernel(Format f, const float *__restrict__ X, int64_t batch, float *__restr
     constexpr int kEsz = BF16 ? 2 : 4;
     extern __shared__ __align__(128) unsigned char sm[];
     Bars &bar = *reinterpret_cast<Bars *>(sm);
-    float *s_x = reinterpret_cast<float *>(sm + 128);
+    float *s_x = reinterpret_cast<float *>(sm + kBarBytes);
     unsigned char *s_ring = sm + p.ring_off;
     float *s_part = reinterpret_cast<float *>(sm + p.part_off);   // [kMaxGroups * 32 rows][T]
 
@@ -159,7 +166,7 @@ xres_kernel(Format f, const float *__restrict__ X, int64_t batch, float *__restr
             mbar_init(&bar.full[st], 1);
             mbar_init(&bar.empty[st], kCWarps);
         }
-        mbar_init(&bar.xfull, 1);
+        for (int i = 0; i < p.nboxes; ++i) mbar_init(&bar.xbox[i], 1);
         mbar_init(&bar.xfree, kCWarps);
         mbar_init(&bar.ready, kCWarps * C);   // every consumer warp of every CTA, once a set
         mbar_init(&bar.freed, kRWarps * C);   // every reducer warp of every CTA, once a set
@@ -239,8 +246,31 @@ xres_kernel(Format f, const float *__restrict__ X, int64_t batch, float *__restr
         uint32_t pph = 0u;    // and the parity of its use ((rc / NS) & 1)
         int xloads = 0;       // slices loaded
         int cur_tile = -1;
+        // the boxes of tile `tile`'s slice, each completing its own barrier.  A
+        // box no round needed (past the matrix) may not have been waited for:
+        // every box of the previous slice has landed before a box is reused,
+        // so that the phases of a box's barrier never overlap
+        // (false, nothing issued, if one of them did not land in time)
+        auto load_slice = [&](int tile) {
+            bool drained = true;
+            if (lane == 0 && xloads > 0)
+                for (int i = 0; i < p.nboxes; ++i) drained = mbar_wait(&bar.xbox[i], (xloads - 1) & 1) && drained;
+            if (__shfl_sync(0xFFFFFFFFu, drained ? 1 : 0, 0) == 0) return false;
+            if (lane == 0) {
+                fence_proxy_async_smem();
+                for (int i = 0; i < p.nboxes; ++i) {
+                    mbar_arrive_expect_tx(&bar.xbox[i], uint32_t(p.box_rows) * T * 4);
+                    tensor2d_g2s(s_x + size_t(i) * p.box_rows * T, &xmap, tile * T, kq0 + i * p.box_rows,
+                                 &bar.xbox[i]);
+                }
+            }
+            ++xloads;
+            cur_tile = tile;
+            return true;
+        };
         Cursor cu = cursor_at(u_begin), cn = cu;
         advance(cn);
+        if (u_begin < u_end) ok = load_slice(cu.tile);   // the run's first tile is known: no wait for its set
         Set s_next = u_begin < u_end ? load_set(cu.sidx) : Set{};
         for (int u = u_begin; u < u_end && ok; ++u, cu = cn, advance(cn)) {
             const Set s = s_next;
@@ -251,15 +281,8 @@ xres_kernel(Format f, const float *__restrict__ X, int64_t batch, float *__restr
                 if (xloads > 0) ok = mbar_wait(&bar.xfree, (xloads - 1) & 1, false);
                 ok = __shfl_sync(0xFFFFFFFFu, ok ? 1 : 0, 0) != 0;
                 if (!ok) break;
-                if (lane == 0) {
-                    fence_proxy_async_smem();
-                    mbar_arrive_expect_tx(&bar.xfull, p.x_bytes);
-                    for (int i = 0; i < p.nboxes; ++i)
-                        tensor2d_g2s(s_x + size_t(i) * p.box_rows * T, &xmap, g.tile * T, kq0 + i * p.box_rows,
-                                     &bar.xfull);
-                }
-                ++xloads;
-                cur_tile = g.tile;
+                ok = load_slice(g.tile);
+                if (!ok) break;
             }
             const int rw = s.nib ? 1 : 2;
             const int64_t gnch = (s.n + kChunk - 1) / kChunk;   // chunks of a group
@@ -297,7 +320,8 @@ xres_kernel(Format f, const float *__restrict__ X, int64_t batch, float *__restr
                 const int last = rc - k;
                 mbar_wait(&bar.full[last % NS], (last / NS) & 1);
             }
-            if (xloads > 0) mbar_wait(&bar.xfull, (xloads - 1) & 1);
+            if (xloads > 0)
+                for (int i = 0; i < p.nboxes; ++i) mbar_wait(&bar.xbox[i], (xloads - 1) & 1);
         }
     } else if (warp > kProducerWarp) {
         // ------------------------------------------------------------ reducers
@@ -367,6 +391,7 @@ xres_kernel(Format f, const float *__restrict__ X, int64_t batch, float *__restr
         //    one whole activation row.
         bool ok = true;
         int rc = 0, xloads = 0, cur_tile = -1;
+        int nready = 0;       // boxes of the current slice known to have landed
         int cst = 0;          // the stage of round rc (rc % NS)
         uint32_t cph = 0u;    // and the parity of its use ((rc / NS) & 1)
         Cursor cu = cursor_at(u_begin), cn = cu;
@@ -404,9 +429,16 @@ xres_kernel(Format f, const float *__restrict__ X, int64_t batch, float *__restr
             for (int r = 0; r < g.rounds; ++r, ++rc) {
                 const int st = cst;
                 if (ok) ok = mbar_wait(&bar.full[st], cph, false);
+                const int cr0 = g.c0 + r * g.cpr, nchr = min(g.cpr, g.nch - r * g.cpr);
+                // the boxes holding the slice rows this round's blocks can select
+                // (rows below (cr0 + nchr) * 8 * m - kq0), in order
+                const int hi = (cr0 + nchr) * kChunk * s.m - kq0;
+                while (ok && nready < p.nboxes && nready * p.box_rows < hi) {
+                    ok = mbar_wait(&bar.xbox[nready], (xloads - 1) & 1, false);
+                    ++nready;
+                }
                 ok = __shfl_sync(0xFFFFFFFFu, ok ? 1 : 0, 0) != 0;
                 if (ok) {
-                    const int cr0 = g.c0 + r * g.cpr, nchr = min(g.cpr, g.nch - r * g.cpr);
                     const unsigned char *sv = s_ring + size_t(st) * stage_bytes<BF16>();
                     const uint32_t *so = reinterpret_cast<const uint32_t *>(sv + ring_val_bytes<BF16>());
                     for (int lc = 0; lc < nchr; ++lc) {
@@ -482,9 +514,8 @@ xres_kernel(Format f, const float *__restrict__ X, int64_t batch, float *__restr
                     __syncwarp();
                     if (lane == 0) mbar_arrive(&bar.xfree);
                 }
-                if (ok) ok = mbar_wait(&bar.xfull, xloads & 1, false);
-                ok = __shfl_sync(0xFFFFFFFFu, ok ? 1 : 0, 0) != 0;
-                ++xloads;
+                ++xloads;           // its boxes are waited for by the rounds that read them
+                nready = 0;
                 cur_tile = g.tile;
             }
             using L4 = std::integral_constant<int, 4>;
@@ -595,7 +626,8 @@ cudaError_t launch(const Format &f, const float *X, int64_t ldx, int64_t batch, 
         const int nboxes = static_cast<int>((rows + 255) / 256);
         const int box_rows = static_cast<int>((rows + nboxes - 1) / nboxes);
         const uint64_t x_bytes = uint64_t(nboxes) * box_rows * T * 4;
-        const uint64_t ring_off = 128 + x_bytes;
+        if (nboxes > kMaxBoxes) continue;
+        const uint64_t ring_off = kBarBytes + x_bytes;
         const uint64_t part_bytes = uint64_t(kMaxGroups) * kSlots * T * 4;
         if (ring_off + 2 * stage_bytes<BF16>() + part_bytes > kSmemCap) continue;
         const int nst = static_cast<int>(
