@@ -653,10 +653,12 @@ cudaError_t launch(const Format &f, const float *X, int64_t ldx, int64_t batch, 
     }
     if (best_sms <= 0) return cudaErrorNotSupported;
     const int64_t occ = std::min<int64_t>(max_clusters<BF16, T>(p.C, smem), kMaxClusters);
-    // Row sets of about 4 heaviest groups (table 1: 128 rows and more, the
-    // consumers' efficient layout) when they still give every cluster 3 units or
-    // more; else sets of about 2 (table 0), whose finer units balance better.
-    const int table = tiles * f.nxsets[1] >= 3 * occ ? 1 : 0;
+    // Row sets of about 4 heaviest groups (table 1: 128 rows, the consumers'
+    // efficient layout) when they still give every cluster 2 units or more;
+    // else sets of about 2 (table 0), whose finer units balance better.  (At
+    // 3 units a cluster FC6 batch 64 took table 0 on clusters of 6: 20.3
+    // against 18.8 us; at 1, FC7 batch 64 took table 1: 13.8 against 12.8.)
+    const int table = tiles * f.nxsets[1] >= 2 * occ ? 1 : 0;
     const int nsets = f.nxsets[table];
     const int64_t units = tiles * nsets;
     p.table = table;
