@@ -690,25 +690,45 @@ cudaError_t launch(const Format &f, const float *X, int64_t ldx, int64_t batch, 
         cost[static_cast<size_t>(s) + 1] = cost[static_cast<size_t>(s)] + hs[s].ng * most + kUnitCost;
     }
     const int64_t *pre = cost.data();
-    auto unit_cost = [&](int64_t u) {
-        const int64_t sidx = u % nsets;
-        return pre[sidx + 1] - pre[sidx] + (sidx == 0 ? kSwitchCost : 0);
-    };
-    // (the switch is charged to a unit that opens a batch tile inside a run; a
-    // run's own first unit is charged its work alone)
+    // One greedy pass for a bound: a run takes its first unit whatever that
+    // costs, then the following units while they fit, a unit that opens a
+    // tile inside the run carrying kSwitchCost.  Whole tiles are taken at
+    // once and the fitting prefix of a tile is found in the prefix sums, so a
+    // pass costs about one step per tile and per run, not one per unit.
+    const int64_t wt = pre[nsets];   // the units of one tile
     auto greedy = [&](int64_t bound, bool write) {
         int c = 0;
         for (int64_t u = 0; u < units; ++c) {
             const int64_t u0 = u;
-            int64_t acc = pre[u % nsets + 1] - pre[u % nsets];
-            for (++u; u < units && acc + unit_cost(u) <= bound; ++u) acc += unit_cost(u);
+            int64_t sidx = u % nsets;
+            int64_t acc = pre[sidx + 1] - pre[sidx];
+            ++u;
+            ++sidx;
+            while (u < units) {
+                if (sidx == nsets) {   // the next unit opens a tile
+                    if (acc + kSwitchCost + wt <= bound) {
+                        acc += kSwitchCost + wt;
+                        u += nsets;
+                        continue;
+                    }
+                    const int64_t k = std::upper_bound(pre, pre + nsets + 1, bound - acc - kSwitchCost) - pre - 1;
+                    if (k > 0) u += k;
+                    break;
+                }
+                // the largest e with pre[e] - pre[sidx] <= bound - acc (e >= sidx: acc <= bound)
+                const int64_t e = std::upper_bound(pre + sidx, pre + nsets + 1, bound - acc + pre[sidx]) - pre - 1;
+                u += e - sidx;
+                if (e < nsets) break;
+                acc += wt - pre[sidx];
+                sidx = nsets;
+            }
             if (write) p.range[c] = make_int2(static_cast<int>(u0), static_cast<int>(u));
         }
         return c;
     };
-    int64_t lo = 0, hi = 0;
+    int64_t lo = 0;
     for (int sidx = 0; sidx < nsets; ++sidx) lo = std::max<int64_t>(lo, pre[sidx + 1] - pre[sidx]);
-    for (int64_t u = 0; u < units; ++u) hi += unit_cost(u);
+    int64_t hi = tiles * (wt + kSwitchCost);   // one run of everything fits
     while (lo < hi) {   // the smallest bound whose runs fit ncl clusters
         const int64_t mid = lo + (hi - lo) / 2;
         if (greedy(mid, false) <= ncl) hi = mid;
