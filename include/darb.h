@@ -138,6 +138,23 @@ DARB_API darb_status_t darb_encode(const void *W, darb_dtype_t wtype, int64_t ro
  */
 DARB_API darb_status_t darb_reencode(darb_handle_t h, const void *W, int64_t ldw, cudaStream_t stream);
 
+/*
+ * darb_reencode from weights in HOST memory (Sec. 3.1's BMWM on a W that
+ * lives on the host, as a serving or training loop hands it over).
+ *   W      host, rows x ldw elements of the handle's dtype, row-major,
+ *          ldw >= cols; only the first cols of each row are read.
+ *   W_dev  device, rows x ldw elements (aligned to the element size), owned
+ *          by the caller: W is copied there (rows of cols elements at pitch
+ *          ldw), then re-encoded from it; it keeps the copy afterwards.
+ * The copy and the encode are ordered on `stream`.  With pinned host memory
+ * the call is asynchronous; with pageable memory the copy completes before
+ * the call returns.  Allocates nothing.
+ * Errors: as darb_reencode, and DARB_ERR_INVALID_ARG for a null W_dev;
+ * DARB_ERR_CUDA if the copy cannot be issued.
+ */
+DARB_API darb_status_t darb_reencode_host(darb_handle_t h, const void *W, int64_t ldw, void *W_dev,
+                                          cudaStream_t stream);
+
 /* Synchronise `stream` and report what the handle's kernels recorded on the
  * device since the last call, then clear it: DARB_ERR_TIMEOUT if a bounded
  * device wait (for a bulk copy, or at a sequence call's grid barrier) gave up
@@ -164,6 +181,25 @@ DARB_API darb_status_t darb_sync_status(darb_handle_t h, cudaStream_t stream);
  */
 DARB_API darb_status_t darb_spmm(darb_handle_t h, const float *X, int64_t ldx, int64_t batch, float *Y,
                         int64_t ldy, cudaStream_t stream);
+
+/*
+ * darb_spmm with X and Y in HOST memory (Sec. 3.2's product as a caller
+ * outside the GPU sees it: activations in, outputs back).
+ *   X      host fp32, cols x batch, ldx >= batch.
+ *   Y      host fp32, rows x batch, ldy >= batch; receives the product.
+ *   X_dev  device fp32, cols x batch (rows of batch floats), owned by the
+ *          caller: X is copied there first.
+ *   Y_dev  device fp32, rows x batch (rows of batch floats), owned by the
+ *          caller: the product is written there, then copied into Y.  Must
+ *          not overlap X_dev.
+ * Copy in, product (darb_spmm on X_dev, Y_dev) and copy out are ordered on
+ * `stream`; with pinned host memory the call is asynchronous and Y holds the
+ * product once `stream` has been synchronised.  Allocates nothing.
+ * Errors: as darb_spmm (X_dev and Y_dev checked as its X and Y, X and Y for
+ * null); DARB_ERR_CUDA if a copy cannot be issued.
+ */
+DARB_API darb_status_t darb_spmm_host(darb_handle_t h, const float *X, int64_t ldx, int64_t batch, float *Y,
+                                      int64_t ldy, float *X_dev, float *Y_dev, cudaStream_t stream);
 
 /* Which kernels compute a product (the paper has no counterpart: these are two
  * ways of evaluating the same sum on the GPU).                               */

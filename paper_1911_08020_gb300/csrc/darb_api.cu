@@ -602,6 +602,28 @@ darb_status_t darb_reencode(darb_handle_t h, const void *W, int64_t ldw, cudaStr
     return DARB_OK;
 }
 
+// A host <-> device copy of `rows` rows of `width` bytes, one cudaMemcpyAsync
+// when both sides are contiguous, else one pitched copy.
+static cudaError_t copy_rows(void *dst, size_t dpitch, const void *src, size_t spitch, size_t width, int64_t rows,
+                             cudaMemcpyKind kind, cudaStream_t stream) {
+    if (dpitch == width && spitch == width)
+        return cudaMemcpyAsync(dst, src, width * static_cast<size_t>(rows), kind, stream);
+    return cudaMemcpy2DAsync(dst, dpitch, src, spitch, width, static_cast<size_t>(rows), kind, stream);
+}
+
+darb_status_t darb_reencode_host(darb_handle_t h, const void *W, int64_t ldw, void *W_dev, cudaStream_t stream) {
+    DARB_TRACE("darb_reencode_host");
+    if (!live(h) || W == nullptr || W_dev == nullptr || ldw < h->cols) return DARB_ERR_INVALID_ARG;
+    const size_t esz = h->wtype == DARB_BF16 ? 2 : 4;
+    if (reinterpret_cast<uintptr_t>(W) % esz != 0 || reinterpret_cast<uintptr_t>(W_dev) % esz != 0)
+        return DARB_ERR_INVALID_ARG;
+    const size_t pitch = static_cast<size_t>(ldw) * esz;
+    if (copy_rows(W_dev, pitch, W, pitch, static_cast<size_t>(h->cols) * esz, h->rows, cudaMemcpyHostToDevice,
+                  stream) != cudaSuccess)
+        return DARB_ERR_CUDA;
+    return darb_reencode(h, W_dev, ldw, stream);
+}
+
 darb_status_t darb_sync_status(darb_handle_t h, cudaStream_t stream) {
     DARB_TRACE("darb_sync_status");
     if (!live(h)) return DARB_ERR_INVALID_ARG;
@@ -643,6 +665,31 @@ darb_status_t darb_spmm_ex(darb_handle_t h, const float *X, int64_t ldx, int64_t
         return DARB_ERR_OOM;
     }
     return cuda_status(e);
+}
+
+darb_status_t darb_spmm_host(darb_handle_t h, const float *X, int64_t ldx, int64_t batch, float *Y, int64_t ldy,
+                             float *X_dev, float *Y_dev, cudaStream_t stream) {
+    DARB_TRACE("darb_spmm_host");
+    if (!live(h) || X == nullptr || Y == nullptr || X_dev == nullptr || Y_dev == nullptr || batch <= 0 ||
+        ldx < batch || ldy < batch)
+        return DARB_ERR_INVALID_ARG;
+    if (reinterpret_cast<uintptr_t>(X) % 4 != 0 || reinterpret_cast<uintptr_t>(Y) % 4 != 0 ||
+        reinterpret_cast<uintptr_t>(X_dev) % 4 != 0 || reinterpret_cast<uintptr_t>(Y_dev) % 4 != 0)
+        return DARB_ERR_INVALID_ARG;
+    if (batch > kMaxBatch) return DARB_ERR_UNSUPPORTED;
+    const size_t row = static_cast<size_t>(batch) * 4;
+    // every check before the first copy: a rejected call does no device work
+    if (overlaps(X_dev, row * static_cast<size_t>(h->cols), Y_dev, row * static_cast<size_t>(h->rows)))
+        return DARB_ERR_INVALID_ARG;
+    if (copy_rows(X_dev, row, X, static_cast<size_t>(ldx) * 4, row, h->cols, cudaMemcpyHostToDevice, stream) !=
+        cudaSuccess)
+        return DARB_ERR_CUDA;
+    const darb_status_t st = darb_spmm(h, X_dev, batch, batch, Y_dev, batch, stream);
+    if (st != DARB_OK) return st;
+    if (copy_rows(Y, static_cast<size_t>(ldy) * 4, Y_dev, row, row, h->rows, cudaMemcpyDeviceToHost, stream) !=
+        cudaSuccess)
+        return DARB_ERR_CUDA;
+    return DARB_OK;
 }
 
 darb_status_t darb_assign_from_weights(const void *W, darb_dtype_t wtype, int64_t rows, int64_t cols, int64_t ldw,

@@ -55,9 +55,11 @@ def lib():
                 "darb_assign_from_weights": [P, ctypes.c_int, I64, I64, I64, I64, I32, I32, P, P, S],
                 "darb_encode": [P, ctypes.c_int, I64, I64, I64, P, P, S],
                 "darb_reencode": [P, P, I64, S],
+                "darb_reencode_host": [P, P, I64, P, S],
                 "darb_sync_status": [P, S],
                 "darb_spmm": [P, P, I64, I64, P, I64, S],
                 "darb_spmm_ex": [P, P, I64, I64, P, I64, ctypes.c_int, S],
+                "darb_spmm_host": [P, P, I64, I64, P, I64, P, P, S],
                 "darb_spmm_path": [P, I64, P, P],
                 "darb_lstm_step": [P, I64, I64, I64, P, P, P, P, P, P, S],
                 "darb_lstm_step_noalloc": [P, I64, I64, I64, P, P, P, P, P, P, S],
@@ -182,6 +184,17 @@ def darb_reencode(h: Handle, W, stream=None):
     _check(lib().darb_reencode(h.ptr, _ptr(W), W.stride(0), _stream(stream)), "darb_reencode")
 
 
+def darb_reencode_host(h: Handle, W, W_dev, stream=None):
+    """darb_reencode from a host W (CPU tensor, rows x cols, row stride ldw) through
+    the caller's device buffer W_dev (same shape and row stride)."""
+    if W.is_cuda or not W_dev.is_cuda or W.dtype != W_dev.dtype:
+        raise DarbError(ERR_INVALID_ARG, "darb_reencode_host: W on the host, W_dev on the device, one dtype")
+    if W.shape != W_dev.shape or W.stride() != W_dev.stride() or W.stride(1) != 1:
+        raise DarbError(ERR_INVALID_ARG, "darb_reencode_host: W and W_dev of one row-major layout")
+    _check(lib().darb_reencode_host(h.ptr, _ptr(W), W.stride(0), _ptr(W_dev), _stream(stream)),
+           "darb_reencode_host")
+
+
 def darb_sync_status(h: Handle, stream=None):
     """Synchronise and raise if the handle's kernels recorded a NaN or a timeout."""
     _check(lib().darb_sync_status(h.ptr, _stream(stream)), "darb_sync_status")
@@ -211,6 +224,26 @@ def darb_spmm_ex(h: Handle, X, Y=None, path: int = PATH_AUTO, stream=None):
     else:
         _check(lib().darb_spmm_ex(h.ptr, _ptr(X), ldx, batch, _ptr(Y), ldy, int(path), _stream(stream)),
                "darb_spmm_ex")
+    return Y
+
+
+def darb_spmm_host(h: Handle, X, Y, X_dev, Y_dev, stream=None):
+    """darb_spmm with X (cols x batch) and Y (rows x batch) host float32 tensors
+    (rows strided, columns contiguous) through the caller's dense device buffers
+    X_dev (cols x batch) and Y_dev (rows x batch); returns Y."""
+    import torch
+    for t, n, cuda in ((X, "X", False), (Y, "Y", False), (X_dev, "X_dev", True), (Y_dev, "Y_dev", True)):
+        if t.dtype != torch.float32 or t.is_cuda != cuda or t.dim() != 2 or (t.shape[1] > 1 and t.stride(1) != 1):
+            raise DarbError(ERR_INVALID_ARG, f"darb_spmm_host: {n} must be a 2-D float32 "
+                                             f"{'CUDA' if cuda else 'host'} tensor with contiguous columns")
+    batch = X.shape[1]
+    if (X_dev.shape != X.shape or Y.shape != (h.rows, batch) or Y_dev.shape != Y.shape or
+            not X_dev.is_contiguous() or not Y_dev.is_contiguous()):
+        raise DarbError(ERR_INVALID_ARG, "darb_spmm_host: shapes, or device buffers not dense")
+    ldx = X.stride(0) if X.shape[0] > 1 else batch
+    ldy = Y.stride(0) if Y.shape[0] > 1 else batch
+    _check(lib().darb_spmm_host(h.ptr, _ptr(X), ldx, batch, _ptr(Y), ldy, _ptr(X_dev), _ptr(Y_dev),
+                                _stream(stream)), "darb_spmm_host")
     return Y
 
 

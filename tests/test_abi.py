@@ -126,6 +126,8 @@ def test_calls_reject_unknown_handles(L):
     assert L.darb_gru_sequence(bogus, 2, 1, 1, 1, 4096, 4096, None, None, 8192, None) == darb.ERR_INVALID_ARG
     assert L.darb_export(bogus, None, None, None, None) == darb.ERR_INVALID_ARG
     assert L.darb_reencode(bogus, 4096, 8, None) == darb.ERR_INVALID_ARG
+    assert L.darb_reencode_host(bogus, 4096, 8, 8192, None) == darb.ERR_INVALID_ARG
+    assert L.darb_spmm_host(bogus, 4096, 1, 1, 8192, 1, 12288, 16384, None) == darb.ERR_INVALID_ARG
     assert L.darb_rnn_reserve(bogus, 4) == darb.ERR_INVALID_ARG
     assert L.darb_destroy(bogus) == darb.ERR_INVALID_ARG
     assert L.darb_destroy(None) == darb.OK
