@@ -128,13 +128,18 @@ template <> struct Packed<false> {  // fp32 bits, index
     static __device__ __forceinline__ uint32_t col(T w) { return w.y; }
 };
 
-// Grid-wide barrier with a time limit (the arrive/spin/fence pattern of a
-// cooperative grid sync); false if this CTA gave up or another CTA did.
+// Grid-wide barrier with a time limit; false if this CTA gave up or another
+// CTA did.  The CTA barrier orders every thread's h_t stores before thread 0's
+// arrival, a release reduction on the counter (no return trip, no separate
+// fence); thread 0 then polls with acquire loads.  An acquire that reads the
+// final count synchronises with every arrival (each is a read-modify-write in
+// the counter's release sequence), and the closing CTA barrier carries that
+// to the CTA's other threads.
 __device__ __forceinline__ bool grid_barrier(const SeqArgs &a, unsigned target, int *s_ok) {
     __syncthreads();
     if (threadIdx.x == 0) {
-        __threadfence();   // the CTA's h_t stores are visible before its arrival counts
-        if (!(int(blockIdx.x) == a.skip_cta && target == gridDim.x)) atomicAdd(a.bar, 1u);
+        if (!(int(blockIdx.x) == a.skip_cta && target == gridDim.x))
+            asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(a.bar) : "memory");
         int ok = 1;
         const unsigned long long t0 = global_timer_ns();
         for (unsigned spin = 0;; ++spin) {
@@ -155,7 +160,6 @@ __device__ __forceinline__ bool grid_barrier(const SeqArgs &a, unsigned target, 
                 __nanosleep(32);
             }
         }
-        __threadfence();
         *s_ok = ok;
     }
     __syncthreads();
