@@ -112,7 +112,7 @@ __host__ __device__ constexpr uint32_t stage_bytes() { return ring_val_bytes<BF1
 struct Plan {
     int C;            // CTAs per cluster = column slices (1 .. 8)
     int S;            // a slice's blocks start in columns [q*S, (q+1)*S)
-    int nst;          // stages of the ring (kMinStages or fewer only when nothing else fits)
+    int nst;          // stages of the ring (fewer than kMinStages only when nothing else fits)
     int box_rows;     // activation rows per tensor-map box
     int nboxes;       // boxes per slice
     int table;        // row-set table (SetGeo) of the handle
