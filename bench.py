@@ -1047,6 +1047,52 @@ def cpu_protocol(runs: int = 5):
     return out
 
 
+def cpu_configs(runs: int = 3):
+    """The oracle as it stands on the other four configs, at 1 thread and at
+    nproc threads (median of `runs` after one untimed run): config 1's encode
+    (fp32) plus its batch-1 product, and one fp64 cell step of each RNN
+    workload's first layer (the unit the `rnn` section's per-step times use)."""
+    import oracle
+    from paper_1911_08020_gb300 import synth
+    oracle.build()
+    nproc = os.cpu_count() or 1
+    cases = {}
+    wl = synth.WORKLOADS["gemv_1024"]
+    _, stored, m = synth.matrix(wl, 0)
+    x1 = synth.activations(wl.shapes[0][1], 1, seed=wl.seed)
+    cases["gemv_1024"] = (lambda: oracle.darb_spmm_f32(oracle.encode(stored, m, wl.dtype), x1),
+                          "oracle encode (fp32) + darb_spmm_f32 at batch 1")
+    for name, batches in (("lstm_1024", (1, 32)), ("lstm_lm_1500", (20,)), ("gru_1024", (64,))):
+        wr = synth.WORKLOADS[name]
+        _, st_r, m_r = synth.matrix(wr, 0)
+        enc = oracle.encode(st_r, m_r, wr.dtype)
+        I, H = wr.input_size, wr.hidden
+        for B in batches:
+            x, h0 = synth.activations(I, B, seed=1), synth.state(H, B, seed=2)
+            if wr.kind == "lstm":
+                c0 = synth.state(H, B, seed=3, scale=1.0)
+                fn = (lambda enc=enc, I=I, H=H, x=x, h0=h0, c0=c0: oracle.lstm_step(enc, I, H, x, h0, c0))
+            else:
+                fn = (lambda enc=enc, I=I, H=H, x=x, h0=h0: oracle.gru_step(enc, I, H, x, h0))
+            cases[f"{name}_b{B}"] = (fn, f"one oracle {wr.kind} cell step (fp64), first layer")
+    out = {"cpu_model": cpu_model(), "nproc": nproc, "runs": runs}
+    for key, (fn, what) in cases.items():
+        entry = {"sample": what}
+        for threads in (1, nproc):
+            used = oracle.set_threads(threads)
+            fn()
+            times = []
+            for _ in range(runs):
+                t0 = time.perf_counter()
+                fn()
+                times.append(time.perf_counter() - t0)
+            entry["threads_1" if threads == 1 else "threads_nproc"] = {
+                "threads": used, "us": round(statistics.median(times) * 1e6, 1)}
+        out[key] = entry
+    oracle.set_threads(nproc)
+    return out
+
+
 def run_reference(args, world, rank):
     """The reference arm: the CPU oracle as it stands (the paper ships no code)
     runs the GPU arm's step at nproc threads; `value` = the step's algorithmic
@@ -1094,6 +1140,9 @@ def main():
                                    "sample": cp["sample"], "cpu_model": cp["cpu_model"],
                                    "threads_1": cp["threads_1"], "threads_nproc": cp["threads_nproc"],
                                    "same_step_as_gpu": True}
+            if "rnn" in res or "gemv_1024" in res:
+                # the GPU numbers of configs 1-4 are in `gemv_1024` and `rnn`
+                res["cpu_configs"] = cpu_configs()
         print(json.dumps(res), flush=True)
     if world > 1:
         import torch.distributed as dist
