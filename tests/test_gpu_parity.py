@@ -229,6 +229,25 @@ def test_spmm_wide_column_slices(dtype):
             darb.darb_destroy(h)
 
 
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_spmm_too_wide_for_resident_slices(dtype):
+    """Matrices whose activation slice does not fit shared memory even split 8
+    ways (tens of thousands of columns) take the staged-rounds kernel at every
+    batch; products still match the oracle, ragged tiles included."""
+    g = np.random.default_rng(26)
+    for rows, cols, mset in ((100, 20000, (16, 64)), (70, 30000, (5, 32, 256))):
+        stored, m = _random_case(g, rows, cols, dtype, mset)
+        h, ref = encode_both(stored, m, dtype)
+        try:
+            for B in (17, 40, 100):
+                X = synth.activations(cols, B, seed=B + 7)
+                Y = darb.darb_spmm(h, t(X)).cpu().numpy()
+                Yr, A = oracle.darb_spmm(ref, X, with_absdot=True)
+                assert_product_close(Y, Yr, A, TOL[dtype])
+        finally:
+            darb.darb_destroy(h)
+
+
 def test_spmm_leading_dimensions_and_alignment():
     g = np.random.default_rng(21)
     rows, cols = 130, 300
